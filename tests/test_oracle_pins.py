@@ -1,0 +1,341 @@
+"""Pins for the oracle: each test checks oracle/ against something other than
+itself (brute force written differently, a library special case, an algebraic
+identity of the paper, an invariant, or a hand-worked value), chosen so that a
+dropped term, a wrong sign or index, or a transposed operand fails one of them.
+CPU only."""
+import itertools
+import json
+import os
+from fractions import Fraction
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+rng = np.random.default_rng(1234)
+
+
+# ------------------------------------------------------------------ helpers
+
+def scatter_conv(x, w, stride, pad):
+    """Brute force written as a scatter: every input value adds its products to
+    every output it reaches.  Independent of the oracle's gather loop order."""
+    n, h, wd, c = x.shape
+    m, kh, kw, _ = w.shape
+    oh = (h + 2 * pad[0] - kh) // stride[0] + 1
+    ow = (wd + 2 * pad[1] - kw) // stride[1] + 1
+    out = [[[[0] * m for _ in range(ow)] for _ in range(oh)] for _ in range(n)]
+    for b in range(n):
+        for iy in range(h):
+            for ix in range(wd):
+                for i in range(kh):
+                    ty = iy + pad[0] - i
+                    if ty % stride[0]:
+                        continue
+                    oy = ty // stride[0]
+                    if not 0 <= oy < oh:
+                        continue
+                    for j in range(kw):
+                        tx = ix + pad[1] - j
+                        if tx % stride[1]:
+                            continue
+                        ox = tx // stride[1]
+                        if not 0 <= ox < ow:
+                            continue
+                        for o in range(m):
+                            s = 0
+                            for ch in range(c):
+                                s += int(x[b, iy, ix, ch]) * int(w[o, i, j, ch])
+                            out[b][oy][ox][o] += s
+    return np.array(out, dtype=np.int64).reshape(n, oh, ow, m)
+
+
+def im2col(x, kh, kw, stride, pad):
+    """Explicit im2col matrix of Sec. III-B: one row per output pixel, columns in (i, j, c) order."""
+    n, h, wd, c = x.shape
+    xp = np.zeros((n, h + 2 * pad[0], wd + 2 * pad[1], c), np.int64)
+    xp[:, pad[0]:pad[0] + h, pad[1]:pad[1] + wd, :] = x
+    oh = (h + 2 * pad[0] - kh) // stride[0] + 1
+    ow = (wd + 2 * pad[1] - kw) // stride[1] + 1
+    rows = []
+    for b in range(n):
+        for oy in range(oh):
+            for ox in range(ow):
+                patch = xp[b, oy * stride[0]:oy * stride[0] + kh, ox * stride[1]:ox * stride[1] + kw, :]
+                rows.append(patch.reshape(-1))
+    return np.array(rows), (n, oh, ow)
+
+
+def rand_layer(n, h, w, c, m, k, bits=8):
+    x = rng.integers(0, 1 << bits, size=(n, h, w, c))
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, k, k, c))
+    return x, wt
+
+
+def requant_ref(acc, bias, kappa, lam, s, bits):
+    """Compression with exact rationals: floor(((acc+bias)*kappa+lam) / 2^s) clipped."""
+    t = Fraction((acc + bias) * kappa + lam, 2 ** s)
+    return min(max(math.floor(t), 0), (1 << bits) - 1)
+
+
+# ------------------------------------------------------------------ MAC core (Eq. 2, Eq. 6)
+
+@pytest.mark.parametrize("k,stride,pad", [(1, 1, 0), (3, 1, 1), (3, 2, 1), (5, 1, 2), (3, 1, 0), (5, 2, 2),
+                                          (3, 2, 0), (1, 2, 0), (3, 1, 2)])
+def test_conv_acc_matches_scatter_brute_force(k, stride, pad):
+    n, h, w, c, m = 2, 5, 4, 3, 4
+    if k > h + 2 * pad:
+        pytest.skip("kernel larger than padded input")
+    x, wt = rand_layer(n, h, w, c, m, k)
+    got = oracle.conv_acc(x, wt, (stride, stride), (pad, pad))
+    want = scatter_conv(x, wt, (stride, stride), (pad, pad))
+    np.testing.assert_array_equal(got, want)
+
+
+def test_conv_acc_rectangular_stride_pad():
+    x, wt = rand_layer(1, 5, 6, 2, 3, 3)
+    wt = wt[:, :, :2, :]  # 3x2 kernel
+    got = oracle.conv_acc(x, wt, (2, 1), (1, 0))
+    want = scatter_conv(x, wt, (2, 1), (1, 0))
+    np.testing.assert_array_equal(got, want)
+
+
+@pytest.mark.parametrize("k,stride,pad", [(3, 1, 1), (5, 1, 2), (3, 2, 1), (1, 1, 0)])
+def test_conv_acc_matches_torch_conv2d_float64(k, stride, pad):
+    """Library special case: exact in float64 while |acc| < 2^53."""
+    torch = pytest.importorskip("torch")
+    x, wt = rand_layer(2, 9, 7, 8, 5, k)
+    got = oracle.conv_acc(x, wt, (stride, stride), (pad, pad))
+    xt = torch.from_numpy(x.astype(np.float64)).permute(0, 3, 1, 2)
+    wtt = torch.from_numpy(wt.astype(np.float64)).permute(0, 3, 1, 2)
+    want = torch.nn.functional.conv2d(xt, wtt, stride=stride, padding=pad).permute(0, 2, 3, 1).numpy()
+    np.testing.assert_array_equal(got, want.astype(np.int64))
+
+
+def test_im2col_times_weights_equals_direct_conv():
+    """Eq. 6: O(m,x,y) = dot(W(m), im2col(x,y)) with W(m) stored in im2col order."""
+    x, wt = rand_layer(2, 6, 5, 4, 6, 3)
+    cols, (n, oh, ow) = im2col(x, 3, 3, (1, 1), (1, 1))
+    via_matmul = (cols @ wt.reshape(wt.shape[0], -1).T.astype(np.int64)).reshape(n, oh, ow, -1)
+    np.testing.assert_array_equal(oracle.conv_acc(x, wt, (1, 1), (1, 1)), via_matmul)
+
+
+def test_adjacent_pixels_share_weights_eq7():
+    """Eq. 7: output (x+1, y) uses the same W(m) with the next im2col buffer."""
+    x, wt = rand_layer(1, 6, 6, 4, 3, 3)
+    acc = oracle.conv_acc(x, wt, (1, 1), (0, 0))
+    cols, _ = im2col(x, 3, 3, (1, 1), (0, 0))
+    cols = cols.reshape(4, 4, -1)
+    for o in range(3):
+        bank = wt[o].reshape(-1)
+        assert acc[0, 2, 1, o] == int(np.dot(bank, cols[2, 1]))
+        assert acc[0, 2, 2, o] == int(np.dot(bank, cols[2, 2]))
+
+
+def test_linearity_in_weights_and_inputs():
+    x1, w1 = rand_layer(1, 5, 5, 4, 3, 3)
+    x2, w2 = rand_layer(1, 5, 5, 4, 3, 3)
+    a = lambda x, w: oracle.conv_acc(x, w, (1, 1), (1, 1))
+    np.testing.assert_array_equal(a(x1, w1 + w2), a(x1, w1) + a(x1, w2))
+    np.testing.assert_array_equal(a(x1 + x2, w1), a(x1, w1) + a(x2, w1))
+
+
+def test_translation_equivariance_away_from_border():
+    x, wt = rand_layer(1, 8, 8, 3, 2, 3)
+    shifted = np.zeros_like(x)
+    shifted[:, 1:, 2:, :] = x[:, :-1, :-2, :]
+    a = oracle.conv_acc(x, wt, (1, 1), (1, 1))
+    b = oracle.conv_acc(shifted, wt, (1, 1), (1, 1))
+    np.testing.assert_array_equal(b[:, 2:7, 3:7, :], a[:, 1:6, 1:5, :])
+
+
+# ------------------------------------------------------------------ compression (Sec. III-A)
+
+def test_floor_shift_is_floor_division():
+    for t in [-9, -8, -7, -1, 0, 1, 7, 8, 9, -(1 << 40) - 3, (1 << 45) + 5, -(1 << 62)]:
+        for s in [0, 1, 2, 3, 31, 32, 40, 62]:
+            assert oracle.floor_shift(t, s) == math.floor(Fraction(t, 2 ** s))
+
+
+def test_requant_matches_rational_definition():
+    cases = itertools.product([-300000, -5, 0, 7, 123456, (1 << 31) - 5000], [-4096, 0, 4096],
+                              [1, 64, -3, 32767, -32768], [-(1 << 15), 0, 1 << 15], [0, 1, 12, 31, 40, 62],
+                              [8, 4, 2])
+    for acc, bias, kappa, lam, s, bits in cases:
+        assert oracle.requant(acc, bias, kappa, lam, s, bits) == requant_ref(acc, bias, kappa, lam, s, bits)
+
+
+def test_requant_special_cases():
+    # kappa = 2^s, lambda = 0, bias = 0 -> clip(acc)
+    for acc in [-10, 0, 5, 200, 255, 256, 100000]:
+        assert oracle.requant(acc, 0, 1 << 6, 0, 6, 8) == min(max(acc, 0), 255)
+    # kappa = 1, lambda = 0, s = 0 -> saturating ReLU
+    for acc in [-1, 0, 1, 14, 15, 16]:
+        assert oracle.requant(acc, 0, 1, 0, 0, 4) == min(max(acc, 0), 15)
+    # negative t -> 0 ; t >= 2^Q * 2^s -> 2^Q - 1
+    assert oracle.requant(-1, 0, 1, 0, 0, 8) == 0
+    assert oracle.requant(1 << 20, 0, 1, 0, 12, 8) == 255
+    assert oracle.requant((1 << 20) - 1, 0, 1, 0, 12, 8) == 255
+    assert oracle.requant((255 << 12), 0, 1, 0, 12, 8) == 255
+    assert oracle.requant((255 << 12) - 1, 0, 1, 0, 12, 8) == 254
+    # bias is added before kappa: (acc + bias) * kappa, not acc * kappa + bias
+    assert oracle.requant(10, 5, 3, 0, 0, 8) == 45
+
+
+def full_layer_ref(x, wt, bias, kappa, lam, shifts, bits, stride, pad):
+    acc = scatter_conv(x, wt, stride, pad)
+    out = np.empty(acc.shape, np.int64)
+    for idx in np.ndindex(acc.shape):
+        o = idx[-1]
+        out[idx] = requant_ref(int(acc[idx]), int(bias[o]), int(kappa[o]), int(lam[o]), int(shifts[o]), bits)
+    return out
+
+
+@pytest.mark.parametrize("bits", [8, 4, 2])
+def test_full_layer_against_independent_reference(bits):
+    n, h, w, c, m, k = 2, 5, 5, 8, 8, 3
+    x, wt = rand_layer(n, h, w, c, m, k, bits)
+    bias = rng.integers(-50, 50, m)
+    kappa = rng.integers(-5, 40, m)
+    lam = rng.integers(-300, 300, m)
+    shifts = rng.integers(0, 8, m)
+    want = full_layer_ref(x, wt, bias, kappa, lam, shifts, bits, (1, 1), (1, 1))
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=k, kw=k, sh=1, sw=1, ph=1, pw=1, bits=bits)
+    xp = oracle.pack(x.reshape(-1), bits)
+    wp = oracle.pack(wt.reshape(-1), bits)
+    y = oracle.conv_hwc(xp, wp, shape, bias, kappa, lam, shifts=shifts)
+    got = oracle.unpack(y, want.size, bits, False).reshape(want.shape)
+    np.testing.assert_array_equal(got, want)
+    # spot pixels through the per-pixel entry point
+    pix = [(0, 0, 0), (1, 4, 4), (1, 2, 3)]
+    yp = oracle.conv_hwc_pixels(xp, wp, shape, bias, kappa, lam, pix, shifts=shifts)
+    for r, (b, oy, ox) in enumerate(pix):
+        np.testing.assert_array_equal(yp[r], want[b, oy, ox])
+
+
+def test_zero_weights_give_bias_only_output():
+    n, h, w, c, m = 1, 4, 4, 8, 4
+    x, _ = rand_layer(n, h, w, c, m, 3)
+    wt = np.zeros((m, 3, 3, c), np.int64)
+    bias = np.array([100, -100, 3000, 7])
+    kappa = np.array([3, 2, 1, -1])
+    lam = np.array([10, 0, -5, 1000])
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=3, kw=3, sh=1, sw=1, ph=1, pw=1, bits=8)
+    y = oracle.conv_hwc(x.reshape(-1), wt.reshape(-1).astype(np.int8).view(np.uint8), shape, bias, kappa, lam,
+                        shift=2).reshape(n, h, w, m)
+    for o in range(m):
+        expect = min(max(math.floor(Fraction(int(bias[o]) * int(kappa[o]) + int(lam[o]), 4)), 0), 255)
+        assert np.all(y[..., o] == expect)
+
+
+def test_centred_one_hot_kernel_copies_a_channel():
+    n, h, w, c, m = 2, 6, 5, 8, 3
+    x, _ = rand_layer(n, h, w, c, m, 3)
+    wt = np.zeros((m, 3, 3, c), np.int64)
+    src = [5, 0, 7]
+    for o, ch in enumerate(src):
+        wt[o, 1, 1, ch] = 1
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=3, kw=3, sh=1, sw=1, ph=1, pw=1, bits=8)
+    y = oracle.conv_hwc(x.reshape(-1), wt.reshape(-1).astype(np.int8).view(np.uint8), shape,
+                        np.zeros(m), np.ones(m), np.zeros(m), shift=0).reshape(n, h, w, m)
+    for o, ch in enumerate(src):
+        np.testing.assert_array_equal(y[..., o], x[..., ch])
+
+
+def test_int4_layer_equals_int8_oracle_on_unpacked_values():
+    """Cross bit-width: the INT-4 path is the INT-8 convolution of the unpacked values, clipped at 15."""
+    n, h, w, c, m = 1, 5, 5, 8, 4
+    x, wt = rand_layer(n, h, w, c, m, 3, bits=4)
+    bias, kappa, lam = rng.integers(-20, 20, m), rng.integers(1, 9, m), rng.integers(-50, 50, m)
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=3, kw=3, sh=1, sw=1, ph=1, pw=1, bits=4)
+    y4 = oracle.conv_hwc(oracle.pack(x.reshape(-1), 4), oracle.pack(wt.reshape(-1), 4), shape, bias, kappa, lam,
+                         shift=3)
+    y4 = oracle.unpack(y4, n * h * w * m, 4, False)
+    shape8 = dict(shape, bits=8)
+    y8 = oracle.conv_hwc(x.reshape(-1).astype(np.uint8), wt.reshape(-1).astype(np.int8).view(np.uint8), shape8,
+                         bias, kappa, lam, shift=3)
+    np.testing.assert_array_equal(y4, np.minimum(y8, 15))
+
+
+def test_accumulator_outside_int32_is_rejected():
+    c = 70000  # 255 * 127 * 70000 > 2^31
+    x = np.full((1, 1, 1, c), 255, np.uint8)
+    wt = np.full((1, 1, 1, c), 127, np.int8)
+    shape = dict(n=1, h=1, w=1, c=c, m=1, kh=1, kw=1, sh=1, sw=1, ph=0, pw=0, bits=8)
+    with pytest.raises(OverflowError):
+        oracle.conv_hwc(x.reshape(-1), wt.reshape(-1).view(np.uint8), shape, np.zeros(1), np.ones(1),
+                        np.zeros(1), shift=0)
+
+
+# ------------------------------------------------------------------ packing (Sec. IV-A)
+
+def test_packing_worked_bytes():
+    with open(os.path.join(GOLDEN, "packing_worked_bytes.json")) as f:
+        cases = json.load(f)["cases"]
+    for case in cases:
+        got = oracle.pack(np.array(case["values"]), case["bits"])
+        assert list(got) == case["bytes"], case
+        back = oracle.unpack(np.array(case["bytes"], np.uint8), len(case["values"]), case["bits"], case["signed"])
+        assert list(back) == case["values"], case
+
+
+@pytest.mark.parametrize("bits", [8, 4, 2])
+@pytest.mark.parametrize("signed", [False, True])
+def test_pack_unpack_round_trip_over_all_bytes(bits, signed):
+    allbytes = np.arange(256, dtype=np.uint8)
+    per = 8 // bits
+    vals = oracle.unpack(allbytes, 256 * per, bits, signed)
+    lo, hi = (-(1 << (bits - 1)), (1 << (bits - 1)) - 1) if signed else (0, (1 << bits) - 1)
+    assert vals.min() >= lo and vals.max() <= hi
+    np.testing.assert_array_equal(oracle.pack(vals, bits), allbytes)
+
+
+# ------------------------------------------------------------------ max-pool and fully connected
+
+def test_maxpool_matches_torch():
+    torch = pytest.importorskip("torch")
+    x = rng.integers(0, 256, size=(2, 8, 6, 16)).astype(np.uint8)
+    y = oracle.maxpool(x.reshape(-1), 2, 8, 6, 16, 2, 2, 8).reshape(2, 4, 3, 16)
+    xt = torch.from_numpy(x.astype(np.float32)).permute(0, 3, 1, 2)
+    want = torch.nn.functional.max_pool2d(xt, 2, 2).permute(0, 2, 3, 1).numpy().astype(np.uint8)
+    np.testing.assert_array_equal(y, want)
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+def test_maxpool_subbyte_matches_unpacked(bits):
+    x = rng.integers(0, 1 << bits, size=(1, 7, 5, 8))
+    y = oracle.maxpool(oracle.pack(x.reshape(-1), bits), 1, 7, 5, 8, 3, 2, bits)
+    got = oracle.unpack(y, 3 * 2 * 8, bits, False).reshape(1, 3, 2, 8)
+    want = np.zeros((1, 3, 2, 8), np.int64)
+    for oy in range(3):
+        for ox in range(2):
+            want[0, oy, ox] = x[0, 2 * oy:2 * oy + 3, 2 * ox:2 * ox + 3].reshape(-1, 8).max(axis=0)
+    np.testing.assert_array_equal(got, want)
+
+
+def test_linear_matches_numpy_int64():
+    x = rng.integers(0, 256, size=(7, 1024)).astype(np.uint8)
+    w = rng.integers(-128, 128, size=(10, 1024)).astype(np.int8)
+    b = rng.integers(-4096, 4097, size=10).astype(np.int32)
+    want = x.astype(np.int64) @ w.astype(np.int64).T + b
+    np.testing.assert_array_equal(oracle.linear(x, w, b), want)
+    np.testing.assert_array_equal(oracle.linear(x, w, None), want - b)
+
+
+def test_paper_benchmark_layer_mac_count():
+    """Sec. V-A layer: 16x16x32 -> 64 filters 3x3x32 is 4,718,592 MACs; an all-ones
+    layer without padding makes every accumulator count its own terms."""
+    with open(os.path.join(GOLDEN, "paper_benchmark_layer.json")) as f:
+        g = json.load(f)
+    h, w, c = g["input_hwc"]
+    m, kh, kw, _ = g["filters_mkkc"]
+    x = np.ones((1, h + 2, w + 2, c), np.int64)  # explicit zero-free padding ring
+    wt = np.ones((m, kh, kw, c), np.int64)
+    acc = oracle.conv_acc(x, wt, (1, 1), (0, 0))
+    assert acc.shape == (1,) + tuple(g["output_hwc"])
+    assert int(acc.sum()) == g["macs"]
+    # the paper's own cycle counts give 13.07 MAC/cycle on 8 cores
+    assert round(g["macs"] / g["table2_cycles_8cores"], 2) == 13.07
