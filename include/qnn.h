@@ -1,0 +1,191 @@
+/*
+ * qnn.h - C ABI of the GB300 (sm_103a) quantized HWC convolution library.
+ *
+ * Method: PULP-NN, "Accelerating Quantized Neural Networks on Parallel
+ * Ultra-Low-Power RISC-V Processors" (arXiv 1908.11263).  The library runs the
+ * data-parallel hot path of that method on one GPU: im2col + integer MatMul
+ * with 32-bit accumulation (Sec. III-B, Eq. 2 and Eq. 6), compression of the
+ * accumulator back to Q bits (Sec. III-A), max-pooling and the fully connected
+ * layer (Sec. IV-A), for INT-8 and packed INT-4 / INT-2 data (Sec. IV-A,
+ * "Sub-byte Extensions").
+ *
+ * Conventions shared by every entry point
+ *  - Plain C types only.  Pointers marked "device" must point to memory of the
+ *    current CUDA device; the caller allocates and owns every buffer, and keeps
+ *    it alive until the work queued on `stream` has finished.
+ *  - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
+ *    stream.  Every call only enqueues work and returns; device-side problems
+ *    surface at the caller's next synchronisation, or through
+ *    qnn_device_status().
+ *  - Arguments are validated before anything is launched; a call that returns
+ *    an error has enqueued nothing.  Nothing is thrown across the ABI.
+ *  - Tensors are dense and contiguous; there are no stride arguments.  Input
+ *    and output buffers must not overlap.
+ *  - Sub-byte storage: element e of a packed Q-bit stream sits in byte
+ *    e / (8/Q) at bits [(e mod (8/Q)) * Q, +Q), the first element in the least
+ *    significant bits.  Activations are unsigned, weights two's-complement.
+ *  - Thread safety: calls may be made from several host threads; the only
+ *    shared host state is a per-device cache of queried device properties.
+ */
+#ifndef QNN_H
+#define QNN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    QNN_OK = 0,
+    QNN_EINVAL = 1,        /* NULL pointer, non-positive size, empty output, shift out of [0,62], bad struct_size */
+    QNN_EUNSUPPORTED = 2,  /* bits not in {8,4,2}; mixed bit-widths; C, M or a count not a whole number of bytes
+                              at Q bits; accumulator bound above int32; forced algorithm that cannot run the shape */
+    QNN_EALIGN = 3,        /* a tensor pointer that must be 16-byte aligned is not */
+    QNN_ECUDA = 4,         /* a CUDA runtime call or kernel launch failed */
+    QNN_ETIMEOUT = 5,      /* a bounded device-side wait gave up (reported by qnn_device_status) */
+    QNN_EWORKSPACE = 6     /* workspace missing or smaller than qconv_hwc_workspace_size() */
+} qnn_status;
+
+/* Convolution algorithm choice (qnn_conv_desc.algo). */
+enum {
+    QNN_ALGO_AUTO = 0,         /* tensor-core kernel when the shape allows it, else the CUDA-core kernel */
+    QNN_ALGO_DIRECT = 1,       /* CUDA-core kernel (dp4a), any stride / padding */
+    QNN_ALGO_TENSORCORE = 2    /* tcgen05 implicit GEMM; QNN_EUNSUPPORTED when the shape does not fit it */
+};
+
+/*
+ * One convolution layer (Sec. III-B).  Input x is NHWC [n][h][w][c]; filters
+ * are [m][kh][kw][c] with c innermost, so each bank W(m) is stored in im2col
+ * order (Eq. 6).  Output y is NHWC [n][oh][ow][m] with
+ * oh = (h + 2*pad_h - kh) / stride_h + 1 and ow likewise (floor).  Padding
+ * reads as activation 0.  x, w and y all use `bits` per element.
+ */
+typedef struct {
+    uint32_t struct_size;      /* = sizeof(qnn_conv_desc) */
+    int32_t n, h, w, c;        /* input batch, height, width, channels; n may be 0 (no work) */
+    int32_t m, kh, kw;         /* output channels, kernel height and width */
+    int32_t stride_h, stride_w;
+    int32_t pad_h, pad_w;
+    int32_t bits;              /* Q in {8, 4, 2} for activations, weights and outputs alike */
+    int32_t shift;             /* right shift in [0, 62], used for every channel when shifts == NULL */
+    int32_t algo;              /* QNN_ALGO_* */
+} qnn_conv_desc;
+
+/*
+ * Bytes of device workspace qconv_hwc() needs for this layer (0 when the
+ * chosen kernel needs none).  The workspace holds the filters re-laid out for
+ * the tensor cores and the per-channel compression constants; it is rewritten
+ * by every call, so one workspace must not be shared by calls that can run
+ * concurrently.
+ */
+qnn_status qconv_hwc_workspace_size(const qnn_conv_desc *d, size_t *bytes);
+
+/*
+ * Quantized convolution with fused compression (Sec. III-A, III-B, IV-A):
+ *
+ *   acc[n][oy][ox][o] = sum_{i<kh, j<kw, ch<c} x[n][oy*sh-ph+i][ox*sw-pw+j][ch] * w[o][i][j][ch]   (int32)
+ *   y[n][oy][ox][o]   = clip( floor( ((acc + bias[o]) * kappa[o] + lambda[o]) / 2^shift_o ), 0, 2^Q - 1 )
+ *
+ * computed exactly (64-bit intermediate for the scaled value); the clip is
+ * also the ReLU.  shift_o = shifts[o] when shifts != NULL, else d->shift.
+ *
+ *   x       device, packed unsigned Q-bit NHWC, 16-byte aligned
+ *   w       device, packed signed Q-bit [m][kh][kw][c], 16-byte aligned
+ *   bias    device int32[m], or NULL for zero
+ *   kappa   device int16[m]
+ *   lambda  device int32[m]
+ *   shifts  device uint8[m] with values in [0, 62], or NULL
+ *   y       device, packed unsigned Q-bit NHWC output, 16-byte aligned
+ *   workspace, workspace_bytes: device scratch of at least
+ *           qconv_hwc_workspace_size() bytes, 256-byte aligned (may be NULL
+ *           when that size is 0)
+ *
+ * Requirements (else QNN_EUNSUPPORTED): c and m multiples of 8/Q, and
+ * kh*kw*c*(2^Q-1)*2^(Q-1) < 2^30, so that the int32 accumulator of Eq. 2 cannot
+ * overflow.  The caller keeps |bias| < 2^30 (bias values are not inspected).
+ */
+qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
+                     const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y,
+                     void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * The two halves of qconv_hwc(), for callers whose filters and compression
+ * constants stay fixed across many calls (inference serving):
+ *
+ * qconv_hwc_prepare: writes into `workspace` the filters re-laid out for the
+ *   tensor cores and the per-channel constants derived from bias, kappa,
+ *   lambda and the shifts (same argument rules as qconv_hwc).  For a
+ *   descriptor that selects the CUDA-core kernel it enqueues nothing.
+ * qconv_hwc_run: the convolution itself, reading a workspace prepared for the
+ *   same descriptor (any other workspace content gives undefined results).
+ *   Only for descriptors that select the tensor-core kernel; otherwise
+ *   QNN_EUNSUPPORTED.
+ * qconv_hwc(...) is exactly qconv_hwc_prepare(...) followed by qconv_hwc_run(...)
+ * on the same stream.
+ */
+qnn_status qconv_hwc_prepare(const qnn_conv_desc *d, const void *w, const int32_t *bias, const int16_t *kappa,
+                             const int32_t *lambda, const uint8_t *shifts, void *workspace, size_t workspace_bytes,
+                             void *stream);
+qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const void *workspace,
+                         size_t workspace_bytes, void *stream);
+
+/* Which kernel qconv_hwc() would run for d: QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE;
+ * negative qnn_status on invalid or unsupported descriptors. */
+int32_t qconv_hwc_algo(const qnn_conv_desc *d);
+
+/*
+ * Fully connected layer (Sec. IV-A, matrix-vector product split over output
+ * neurons in Sec. IV-B), without compression:
+ *   y[b][o] = sum_{i<k} x[b][i] * w[o][i] + bias[o]      (int32 output)
+ *   x    device uint8 [n][k]      (HWC-flattened activations)
+ *   w    device int8  [m][k]
+ *   bias device int32 [m] or NULL
+ *   y    device int32 [n][m]
+ * Requirements: k * 255 * 128 < 2^30 (else QNN_EUNSUPPORTED); the caller keeps |bias| < 2^30.
+ */
+qnn_status qlinear(int32_t n, int32_t k, int32_t m, const uint8_t *x, const int8_t *w, const int32_t *bias,
+                   int32_t *y, void *stream);
+
+/*
+ * Max-pooling (Sec. IV-A): y[b][oy][ox][ch] = max_{i,j<k} x[b][oy*s+i][ox*s+j][ch]
+ * on packed unsigned Q-bit NHWC data, no padding, oh = (h-k)/s + 1 (floor).
+ *   x  device, [n][h][w][c] packed at `bits`;  y  device, [n][oh][ow][c] packed at `bits`
+ * Requirements: c a multiple of 8/Q; 1 <= k <= min(h, w); s >= 1.
+ */
+qnn_status qmaxpool(int32_t n, int32_t h, int32_t w, int32_t c, int32_t k, int32_t s, int32_t bits,
+                    const void *x, void *y, void *stream);
+
+/*
+ * Sub-byte packing (Sec. IV-A, "Sub-byte Extensions": two INT-4 or four INT-2
+ * values per byte, and the unpack-to-INT-8 helper of the same section).
+ *   pack_subbyte:   src device int8[count] (the low Q bits of each value are stored),
+ *                   dst device uint8[count*Q/8]
+ *   unpack_subbyte: src device uint8[count*Q/8], dst device int8[count];
+ *                   is_signed != 0 sign-extends (weights), 0 zero-extends (activations)
+ * count must be a multiple of 8/Q; bits in {8,4,2} (8 is a plain copy).
+ */
+qnn_status pack_subbyte(const int8_t *src, void *dst, int64_t count, int32_t bits, void *stream);
+qnn_status unpack_subbyte(const void *src, int8_t *dst, int64_t count, int32_t bits, int32_t is_signed,
+                          void *stream);
+
+/*
+ * Synchronises `stream`, then returns and clears the library's device status
+ * word: QNN_OK, or QNN_ETIMEOUT when a bounded wait inside a kernel gave up
+ * (the kernel then skipped its remaining work and returned).  QNN_ECUDA when
+ * the synchronisation itself fails.
+ */
+qnn_status qnn_device_status(void *stream);
+
+/* Static description of a status code. */
+const char *qnn_status_string(qnn_status s);
+
+/* Library version, for ABI checks: major * 10000 + minor * 100 + patch. */
+int32_t qnn_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QNN_H */

@@ -1,0 +1,69 @@
+// Host-side interfaces between the C ABI (capi.cu) and the kernel files.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace qnn {
+
+struct ConvShape {
+    int n, h, w, c, m, kh, kw, sh, sw, ph, pw, bits, oh, ow;
+};
+
+struct ConvParams {
+    const uint8_t *x;
+    const uint8_t *w;
+    const int32_t *bias;    // may be null
+    const int16_t *kappa;
+    const int32_t *lambda;
+    const uint8_t *shifts;  // may be null
+    int shift;
+    uint8_t *y;
+};
+
+// ---- CUDA-core convolution (any stride / padding) -- conv_direct.cu
+cudaError_t launch_conv_direct(const ConvShape &s, const ConvParams &p, cudaStream_t st);
+
+// ---- tensor-core implicit GEMM (stride 1) -- conv_tc.cu
+struct TcPlan {
+    bool ok;
+    int nt;             // output channels per tile (MMA N): 16, 32, 64 or 128
+    int n_ntiles;       // ceil(m / nt)
+    int c_pad;          // channels per tap rounded up to 16
+    int cs;             // channels per staged slab
+    int nslab;          // c_pad / cs
+    int k_pad;          // kh * kw * c_pad
+    int p_alloc;        // staged positions per horizontal copy
+    int stages;         // staged slabs in flight
+    int tiles_per_img;  // ceil(oh * ow / 128)
+    long long total_tiles;
+    int mmas_per_tile;  // MMAs (K = 16 each) per tile
+    int chunk_mmas;     // MMAs per exact fp32 accumulator chunk
+    int nchunks;        // chunks per tile
+    uint32_t b_bytes, copy_bytes, stage_bytes, smem_bytes, tmem_cols;
+    size_t workspace_bytes;
+};
+
+TcPlan plan_conv_tc(const ConvShape &s);
+cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
+                                cudaStream_t st);
+cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uint8_t *x, uint8_t *y,
+                               const void *workspace, cudaStream_t st);
+
+// ---- max-pool, fully connected, packing
+cudaError_t launch_maxpool(int n, int h, int w, int c, int k, int s, int bits, const uint8_t *x, uint8_t *y,
+                           cudaStream_t st);
+cudaError_t launch_linear(int n, int k, int m, const uint8_t *x, const int8_t *w, const int32_t *bias, int32_t *y,
+                          cudaStream_t st);
+cudaError_t launch_pack(const int8_t *src, uint8_t *dst, long long count, int bits, cudaStream_t st);
+cudaError_t launch_unpack(const uint8_t *src, int8_t *dst, long long count, int bits, int is_signed,
+                          cudaStream_t st);
+
+// number of SMs of the current device (cached per device)
+int device_sm_count();
+
+// device address of the library's status word on the current device (cached per device; null on failure)
+int *device_status_ptr();
+
+}  // namespace qnn

@@ -1,0 +1,128 @@
+"""C-ABI boundary checks that need no GPU: the library builds and loads, exports
+every function include/qnn.h declares, and rejects invalid arguments before
+launching anything (only argument checks run, no CUDA call is reached)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_1908_11263_gb300 import build as qbuild
+from paper_1908_11263_gb300 import qnn
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "qnn.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    qbuild.build()
+    return qnn.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(\w+)\s*\([^;{]*\)\s*;", text)) - {"sizeof"})
+
+
+def test_header_declares_the_expected_surface():
+    names = declared_functions()
+    for f in ("qconv_hwc", "qlinear", "qmaxpool", "pack_subbyte", "unpack_subbyte", "qconv_hwc_workspace_size"):
+        assert f in names
+
+
+def test_library_exports_every_declared_function(lib):
+    missing = [f for f in declared_functions() if not hasattr(lib, f)]
+    assert not missing, missing
+    assert set(qnn.EXPORTED) <= set(declared_functions())
+
+
+def test_version_and_status_strings(lib):
+    assert lib.qnn_version() == 100
+    for s in range(7):
+        assert qnn.status_string(s) not in ("", "unknown status")
+    assert qnn.status_string(99) == "unknown status"
+
+
+def desc(**kw):
+    base = dict(n=2, h=16, w=16, c=32, m=64, kh=3, kw=3, stride=(1, 1), pad=(1, 1), bits=8, shift=12)
+    base.update(kw)
+    return qnn.conv_desc(base["n"], base["h"], base["w"], base["c"], base["m"], base["kh"], base["kw"],
+                         base["stride"], base["pad"], base["bits"], base["shift"], base.get("algo", 0))
+
+
+FAKE = 0x10000  # 16-byte aligned, never dereferenced: every case below fails validation first
+
+
+def conv_status(lib, d, x=FAKE, w=FAKE, bias=FAKE, kappa=FAKE, lam=FAKE, shifts=None, y=FAKE, ws=FAKE, wsb=1 << 30):
+    P = ctypes.c_void_p
+    return lib.qconv_hwc(ctypes.byref(d), P(x), P(w), P(bias), P(kappa), P(lam), P(shifts), P(y), P(ws),
+                         ctypes.c_size_t(wsb), P(0))
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(h=0), qnn.QNN_EINVAL), (dict(c=-1), qnn.QNN_EINVAL), (dict(m=0), qnn.QNN_EINVAL),
+    (dict(n=-1), qnn.QNN_EINVAL), (dict(stride=(0, 1)), qnn.QNN_EINVAL), (dict(pad=(-1, 0)), qnn.QNN_EINVAL),
+    (dict(h=1, pad=(0, 0)), qnn.QNN_EINVAL),  # kernel taller than the padded input
+    (dict(shift=63), qnn.QNN_EINVAL), (dict(shift=-1), qnn.QNN_EINVAL),
+    (dict(bits=3), qnn.QNN_EUNSUPPORTED), (dict(bits=1), qnn.QNN_EUNSUPPORTED),
+    (dict(bits=4, c=33), qnn.QNN_EUNSUPPORTED), (dict(bits=2, m=62), qnn.QNN_EUNSUPPORTED),
+    (dict(c=40000, kh=1, kw=1, pad=(0, 0)), qnn.QNN_EUNSUPPORTED),  # accumulator bound
+    (dict(algo=7), qnn.QNN_EINVAL), (dict(stride=(2, 2), algo=qnn.ALGO_TENSORCORE), qnn.QNN_EUNSUPPORTED),
+])
+def test_conv_descriptor_validation(lib, kw, code):
+    assert conv_status(lib, desc(**kw)) == code
+
+
+def test_conv_pointer_and_alignment_validation(lib):
+    d = desc()
+    assert conv_status(lib, d, x=0) == qnn.QNN_EINVAL
+    assert conv_status(lib, d, w=0) == qnn.QNN_EINVAL
+    assert conv_status(lib, d, kappa=0) == qnn.QNN_EINVAL
+    assert conv_status(lib, d, lam=0) == qnn.QNN_EINVAL
+    assert conv_status(lib, d, y=0) == qnn.QNN_EINVAL
+    assert conv_status(lib, d, x=FAKE + 8) == qnn.QNN_EALIGN
+    assert conv_status(lib, d, y=FAKE + 1) == qnn.QNN_EALIGN
+    assert conv_status(lib, d, w=FAKE + 4) == qnn.QNN_EALIGN
+    assert conv_status(lib, d, bias=FAKE + 2) == qnn.QNN_EALIGN
+    assert conv_status(lib, d, kappa=FAKE + 1) == qnn.QNN_EALIGN
+    assert conv_status(lib, d, ws=0) == qnn.QNN_EWORKSPACE
+    assert conv_status(lib, d, wsb=16) == qnn.QNN_EWORKSPACE
+    assert conv_status(lib, d, ws=FAKE + 16) == qnn.QNN_EWORKSPACE
+    bad = desc()
+    bad.struct_size = 8
+    assert conv_status(lib, bad) == qnn.QNN_EINVAL
+    assert lib.qconv_hwc(None, *([None] * 8), ctypes.c_size_t(0), None) == qnn.QNN_EINVAL
+
+
+def test_algo_selection_and_workspace(lib):
+    assert qnn.conv_algo(desc()) == qnn.ALGO_TENSORCORE
+    assert qnn.conv_algo(desc(stride=(2, 2))) == qnn.ALGO_DIRECT
+    assert qnn.conv_algo(desc(algo=qnn.ALGO_DIRECT)) == qnn.ALGO_DIRECT
+    assert qnn.workspace_size(desc(algo=qnn.ALGO_DIRECT)) == 0
+    ws = qnn.workspace_size(desc())
+    # fp16 filters (64 x 3*3*32) plus 16 bytes of constants per channel
+    assert ws >= 64 * 288 * 2 + 64 * 16
+    for bits in (4, 2):
+        assert qnn.conv_algo(desc(bits=bits)) == qnn.ALGO_TENSORCORE
+    with pytest.raises(qnn.QnnError):
+        qnn.conv_algo(desc(bits=5))
+
+
+def test_other_entry_points_validate(lib):
+    P = ctypes.c_void_p
+    assert lib.qlinear(-1, 4, 4, P(FAKE), P(FAKE), None, P(FAKE), None) == qnn.QNN_EINVAL
+    assert lib.qlinear(4, 0, 4, P(FAKE), P(FAKE), None, P(FAKE), None) == qnn.QNN_EINVAL
+    assert lib.qlinear(4, 4, 4, None, P(FAKE), None, P(FAKE), None) == qnn.QNN_EINVAL
+    assert lib.qlinear(4, 1 << 20, 4, P(FAKE), P(FAKE), None, P(FAKE), None) == qnn.QNN_EUNSUPPORTED
+    assert lib.qlinear(4, 4, 4, P(FAKE), P(FAKE), None, P(FAKE + 2), None) == qnn.QNN_EALIGN
+    assert lib.qmaxpool(1, 4, 4, 8, 5, 2, 8, P(FAKE), P(FAKE), None) == qnn.QNN_EINVAL
+    assert lib.qmaxpool(1, 4, 4, 8, 2, 0, 8, P(FAKE), P(FAKE), None) == qnn.QNN_EINVAL
+    assert lib.qmaxpool(1, 4, 4, 8, 2, 2, 3, P(FAKE), P(FAKE), None) == qnn.QNN_EUNSUPPORTED
+    assert lib.qmaxpool(1, 4, 4, 3, 2, 2, 4, P(FAKE), P(FAKE), None) == qnn.QNN_EUNSUPPORTED
+    assert lib.pack_subbyte(P(FAKE), P(FAKE), 7, 4, None) == qnn.QNN_EUNSUPPORTED
+    assert lib.pack_subbyte(P(FAKE), P(FAKE), -4, 4, None) == qnn.QNN_EINVAL
+    assert lib.pack_subbyte(P(FAKE), P(FAKE), 8, 6, None) == qnn.QNN_EUNSUPPORTED
+    assert lib.unpack_subbyte(None, P(FAKE), 8, 2, 1, None) == qnn.QNN_EINVAL
+    assert lib.unpack_subbyte(P(FAKE), P(FAKE), 6, 2, 1, None) == qnn.QNN_EUNSUPPORTED

@@ -1,0 +1,284 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the oracle,
+element by element (bit-exact: every result is an integer) on the same seeded
+inputs.  Small shapes span several tiles and ragged tails; the workloads run
+at full size (sampled outputs for the largest layers)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_1908_11263_gb300 import inputs, qnn
+
+from gpu_util import (conv_gpu, conv_oracle, first_mismatch, guarded_output, check_guard, to_dev, pack_gpu,
+                      layer_tensors, THREADS)
+
+pytestmark = pytest.mark.gpu
+ALGOS = [qnn.ALGO_TENSORCORE, qnn.ALGO_DIRECT]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def loaded():
+    qnn.load(build_if_missing=True)
+    torch.cuda.set_device(0)
+
+
+def rand_case(seed, n, h, w, c, m, kh, kw, bits, shift_lo=0, shift_hi=20, per_channel=True, kappa_neg=True):
+    rng = np.random.default_rng(seed)
+    x = rng.integers(0, 1 << bits, size=(n, h, w, c))
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, kh, kw, c))
+    bias = rng.integers(-4096, 4097, size=m).astype(np.int32)
+    kappa = rng.integers(-64 if kappa_neg else 1, 65, size=m).astype(np.int16)
+    lam = rng.integers(-(1 << 15), (1 << 15) + 1, size=m).astype(np.int32)
+    shifts = rng.integers(shift_lo, shift_hi + 1, size=m).astype(np.uint8) if per_channel else None
+    shift = int(rng.integers(shift_lo, shift_hi + 1))
+    return x, wt, bias, kappa, lam, shifts, shift
+
+
+# (n, h, w, c, m, kh, kw, stride, pad, bits): tile multiples, ragged tails, odd widths,
+# channel padding, several slabs and output-channel tiles, rectangular kernels
+SHAPES = [
+    (2, 16, 16, 32, 64, 3, 3, (1, 1), (1, 1), 8),
+    (1, 16, 16, 32, 64, 3, 3, (1, 1), (1, 1), 4),
+    (1, 16, 16, 32, 64, 3, 3, (1, 1), (1, 1), 2),
+    (3, 10, 10, 16, 16, 3, 3, (1, 1), (1, 1), 8),
+    (2, 14, 14, 64, 48, 3, 3, (1, 1), (1, 1), 8),
+    (1, 15, 20, 24, 40, 3, 3, (1, 1), (1, 1), 8),
+    (2, 9, 33, 8, 8, 1, 1, (1, 1), (0, 0), 8),
+    (1, 12, 12, 3, 32, 5, 5, (1, 1), (2, 2), 8),
+    (2, 8, 8, 32, 64, 5, 5, (1, 1), (2, 2), 8),
+    (1, 7, 7, 128, 136, 3, 3, (1, 1), (1, 1), 8),
+    (1, 6, 6, 256, 256, 3, 3, (1, 1), (1, 1), 8),
+    (1, 5, 9, 32, 16, 3, 2, (1, 1), (0, 1), 8),
+    (1, 11, 13, 16, 32, 2, 4, (1, 1), (1, 2), 8),
+    (1, 1, 40, 16, 16, 1, 3, (1, 1), (0, 1), 8),
+    (2, 13, 13, 32, 24, 3, 3, (1, 1), (0, 0), 4),
+    (1, 10, 12, 48, 32, 5, 5, (1, 1), (2, 2), 4),
+    (2, 9, 9, 64, 64, 3, 3, (1, 1), (1, 1), 2),
+    (1, 9, 7, 8, 12, 3, 3, (1, 1), (1, 1), 2),
+    (1, 16, 16, 12, 16, 3, 3, (1, 1), (1, 1), 4),
+    (2, 16, 16, 32, 64, 3, 3, (2, 2), (1, 1), 8),
+    (1, 17, 15, 16, 32, 3, 3, (2, 1), (1, 1), 4),
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: "x".join(str(v) for v in s[:7]) + f"_s{s[7][0]}{s[7][1]}_p{s[8][0]}{s[8][1]}_q{s[9]}")
+def test_conv_random_shapes(shape):
+    n, h, w, c, m, kh, kw, stride, pad, bits = shape
+    x, wt, bias, kappa, lam, shifts, shift = rand_case(hash(shape) & 0xFFFF, n, h, w, c, m, kh, kw, bits)
+    want = conv_oracle(x, wt, bias, kappa, lam, shifts, shift, bits, stride, pad)
+    want_scalar = conv_oracle(x, wt, None, kappa, lam, None, shift, bits, stride, pad)
+    desc = qnn.conv_desc(n, h, w, c, m, kh, kw, stride, pad, bits, shift)
+    for algo in ALGOS:
+        if algo == qnn.ALGO_TENSORCORE and stride != (1, 1):
+            continue
+        got = conv_gpu(x, wt, bias, kappa, lam, shifts, shift, bits, stride, pad, algo)
+        assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
+        got = conv_gpu(x, wt, None, kappa, lam, None, shift, bits, stride, pad, algo)
+        assert first_mismatch(got, want_scalar) is None, (algo, "scalar shift, no bias",
+                                                          first_mismatch(got, want_scalar))
+    if stride == (1, 1):
+        assert qnn.conv_algo(desc) == qnn.ALGO_TENSORCORE
+
+
+@pytest.mark.parametrize("shift", [0, 1, 31, 40, 62])
+def test_conv_shift_extremes(shift):
+    x, wt, bias, kappa, lam, _, _ = rand_case(shift + 7, 1, 8, 8, 32, 32, 3, 3, 8)
+    lam = lam * 1000 if shift > 30 else lam
+    for algo in ALGOS:
+        got = conv_gpu(x, wt, bias, kappa, lam.astype(np.int32), None, shift, 8, (1, 1), (1, 1), algo)
+        want = conv_oracle(x, wt, bias, kappa, lam.astype(np.int32), None, shift, 8, (1, 1), (1, 1))
+        assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
+
+
+@pytest.mark.parametrize("xval,wval", [(0, -128), (255, 127), (255, -128), (0, 127), (128, -128), (1, -1)])
+@pytest.mark.parametrize("c", [256, 2304, 1152])
+def test_exact_accumulation_at_the_bounds(xval, wval, c):
+    """Constant 1x1 layers drive every accumulator chunk to its extreme; with kappa=1,
+    shift=0 and lambda = 100 - acc every output reads 100 only if acc is exact."""
+    n, h, w, m = 1, 4, 32, 16
+    x = np.full((n, h, w, c), xval)
+    wt = np.full((m, 1, 1, c), wval)
+    wt[1::2] = -wt[1::2] - (1 if wval > 0 else 0)  # mix signs across channels (stay inside int8)
+    wt = np.clip(wt, -128, 127)
+    acc = (xval * wt.reshape(m, -1).sum(axis=1)).astype(np.int64)
+    lam = (100 - acc).astype(np.int32)
+    kappa = np.ones(m, np.int16)
+    for algo in ALGOS:
+        got = conv_gpu(x, wt, None, kappa, lam, None, 0, 8, (1, 1), (0, 0), algo)
+        assert np.all(got == 100), (algo, np.unique(got))
+
+
+@pytest.mark.parametrize("bits", [8, 4, 2])
+def test_exact_accumulation_random_long_k(bits):
+    """K = 9 * 256 with random data: outputs compared against the oracle with kappa=1
+    and per-channel lambda centring each channel's accumulators, shift 0."""
+    rng = np.random.default_rng(bits)
+    n, h, w, c, m = 1, 6, 6, 256, 32
+    x = rng.integers(0, 1 << bits, size=(n, h, w, c))
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, 3, 3, c))
+    acc = oracle.conv_acc(x, wt, (1, 1), (1, 1))
+    lam = (128 - np.median(acc.reshape(-1, m), axis=0)).astype(np.int32) if bits == 8 else \
+          ((1 << (bits - 1)) - np.median(acc.reshape(-1, m), axis=0)).astype(np.int32)
+    kappa = np.ones(m, np.int16)
+    want = conv_oracle(x, wt, None, kappa, lam, None, 0, bits, (1, 1), (1, 1))
+    for algo in ALGOS:
+        got = conv_gpu(x, wt, None, kappa, lam, None, 0, bits, (1, 1), (1, 1), algo)
+        assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
+
+
+def test_extreme_values_all_layers():
+    for xval, wval in [(0, 0), (255, 127), (255, -128), (0, -128)]:
+        x = np.full((2, 16, 16, 32), xval)
+        wt = np.full((64, 3, 3, 32), wval)
+        _, _, bias, kappa, lam, shifts, shift = rand_case(xval + wval + 1000, 2, 16, 16, 32, 64, 3, 3, 8)
+        want = conv_oracle(x, wt, bias, kappa, lam, shifts, shift, 8, (1, 1), (1, 1))
+        for algo in ALGOS:
+            got = conv_gpu(x, wt, bias, kappa, lam, shifts, shift, 8, (1, 1), (1, 1), algo)
+            assert first_mismatch(got, want) is None, (xval, wval, algo)
+
+
+def test_empty_batch_is_a_no_op():
+    x = torch.empty((0, 16, 16, 32), dtype=torch.uint8, device="cuda")
+    w = torch.zeros((64, 3, 3, 32), dtype=torch.int8, device="cuda")
+    k = torch.ones(64, dtype=torch.int16, device="cuda")
+    lam = torch.zeros(64, dtype=torch.int32, device="cuda")
+    for algo in ALGOS:
+        y = qnn.conv_hwc(x, w, k, lam, shift=3, bits=8, stride=1, pad=1, algo=algo)
+        assert y.shape == (0, 16, 16, 64)
+    qnn.device_status()
+
+
+# ------------------------------------------------------------------ workloads at full size
+
+def run_workload_layer(key, layer, wl, lid, algos=ALGOS):
+    ld = inputs.make_layer(key, layer, wl, lid)
+    x, wt, bias, kappa, lam, shifts, shift = layer_tensors(ld)
+    st, pd = (layer.stride, layer.stride), (layer.pad, layer.pad)
+    want = conv_oracle(x, wt, bias, kappa, lam, shifts, shift, layer.bits, st, pd)
+    for algo in algos:
+        got = conv_gpu(x, wt, bias, kappa, lam, shifts, shift, layer.bits, st, pd, algo)
+        assert first_mismatch(got, want) is None, (key, algo, first_mismatch(got, want))
+    return want
+
+
+def test_workload_single_layer_batch1():
+    (key, layer, wl, lid), = inputs.single_layer_workload(inputs.WORKLOAD_SINGLE)
+    assert layer.macs == 4718592
+    run_workload_layer(key, layer, wl, lid)
+
+
+def test_workload_single_layer_batch512():
+    (key, layer, wl, lid), = inputs.single_layer_workload(inputs.WORKLOAD_BATCH)
+    assert layer.macs == 2415919104
+    run_workload_layer(key, layer, wl, lid)
+
+
+@pytest.mark.parametrize("which", ["w4_int4", "w4_int2"])
+def test_workload_subbyte(which):
+    for key, layer, wl, lid in inputs.single_layer_workload(inputs.WORKLOAD_SUBBYTE):
+        if key == which:
+            run_workload_layer(key, layer, wl, lid)
+
+
+def sample_pixels(n, oh, ow, count, seed):
+    rng = np.random.default_rng(seed)
+    fixed = [(0, 0, 0), (0, 0, ow - 1), (0, oh - 1, 0), (n - 1, oh - 1, ow - 1), (n - 1, oh // 2, ow // 2),
+             (n // 2, 0, ow // 2), (n // 2, oh - 1, ow // 3)]
+    rand = [(int(rng.integers(n)), int(rng.integers(oh)), int(rng.integers(ow))) for _ in range(count)]
+    return fixed + rand
+
+
+@pytest.mark.parametrize("key", ["w5_56", "w5_28", "w5_14", "w5_1x1"])
+def test_workload_sweep_sampled(key):
+    """Large layers at full batch in the benchmark's launch configuration: every output
+    byte of sampled pixels against the oracle, plus the whole output against the
+    independent CUDA-core kernel."""
+    (k2, layer, wl, lid), = [t for t in inputs.single_layer_workload(inputs.WORKLOAD_SWEEP) if t[0] == key]
+    ld = inputs.make_layer(k2, layer, wl, lid)
+    x, wt, bias, kappa, lam, shifts, shift = layer_tensors(ld)
+    st, pd = (layer.stride, layer.stride), (layer.pad, layer.pad)
+    pix = sample_pixels(layer.n, layer.oh, layer.ow, 40, lid)
+    want = oracle.conv_hwc_pixels(x.astype(np.uint8).reshape(-1), wt.astype(np.int8).reshape(-1).view(np.uint8),
+                                  layer.shape(), bias, kappa, lam, pix, shifts=shifts, shift=shift)
+    outs = {}
+    for algo in ALGOS:
+        got = conv_gpu(x, wt, bias, kappa, lam, shifts, shift, 8, st, pd, algo)
+        g = got.reshape(layer.n, layer.oh, layer.ow, layer.m)
+        for r, (b, oy, ox) in enumerate(pix):
+            np.testing.assert_array_equal(g[b, oy, ox], want[r], err_msg=f"{key} algo {algo} pixel {(b, oy, ox)}")
+        outs[algo] = got
+    assert first_mismatch(outs[qnn.ALGO_TENSORCORE], outs[qnn.ALGO_DIRECT]) is None
+
+
+def test_workload_cifar_pipeline():
+    """The CIFAR-10-shaped network (Sec. V-E shape) at batch 1024: three conv layers with
+    2x2 max-pooling and the fully connected layer, GPU chain vs oracle chain."""
+    n = 1024
+    x = inputs.cifar_input(n)
+    xd = to_dev(x)
+    xo = x.reshape(-1)
+    for key, layer, wl, lid in inputs.cifar_layers(n):
+        ld = inputs.make_layer(key, layer, wl, lid, x=np.zeros(1))
+        kappa, lam, bias = to_dev(ld.kappa, torch.int16), to_dev(ld.lam, torch.int32), to_dev(ld.bias, torch.int32)
+        yd = qnn.conv_hwc(xd, to_dev(ld.w), kappa, lam, bias=bias, shift=ld.shift, bits=8, stride=1, pad=layer.pad)
+        xd = qnn.maxpool(yd, 2, 2, 8)
+        yo = oracle.conv_hwc(xo, ld.w.reshape(-1).view(np.uint8), layer.shape(), ld.bias, ld.kappa, ld.lam,
+                             shift=ld.shift, nthreads=THREADS)
+        np.testing.assert_array_equal(yd.cpu().numpy().reshape(-1), yo, err_msg=key)
+        xo = oracle.maxpool(yo, n, layer.oh, layer.ow, layer.m, 2, 2, 8)
+        np.testing.assert_array_equal(xd.cpu().numpy().reshape(-1), xo, err_msg=key + " pool")
+    wfc, bfc = inputs.cifar_fc()
+    yd = qnn.linear(xd.view(n, -1), to_dev(wfc), to_dev(bfc))
+    yo = oracle.linear(xo.reshape(n, -1), wfc, bfc)
+    np.testing.assert_array_equal(yd.cpu().numpy(), yo)
+    qnn.device_status()
+
+
+# ------------------------------------------------------------------ max-pool, FC, packing
+
+@pytest.mark.parametrize("bits,c,k,s", [(8, 32, 2, 2), (8, 64, 3, 2), (8, 24, 2, 2), (8, 5, 2, 1), (4, 32, 2, 2),
+                                        (2, 16, 3, 3), (4, 6, 2, 2)])
+def test_maxpool_parity(bits, c, k, s):
+    rng = np.random.default_rng(c * k + bits)
+    n, h, w = 3, 11, 9
+    x = rng.integers(0, 1 << bits, size=(n, h, w, c))
+    xp = oracle.pack(x.reshape(-1), bits) if bits < 8 else x.astype(np.uint8).reshape(-1)
+    want = oracle.maxpool(xp, n, h, w, c, k, s, bits)
+    xd = pack_gpu(x, bits).view(n, h, w, c * bits // 8)
+    oh, ow = (h - k) // s + 1, (w - k) // s + 1
+    out, buf = guarded_output((n, oh, ow, c * bits // 8))
+    qnn.maxpool(xd, k, s, bits, out=out)
+    check_guard(buf)
+    np.testing.assert_array_equal(out.cpu().numpy().reshape(-1), want)
+
+
+@pytest.mark.parametrize("n,k,m", [(1024, 1024, 10), (5, 7, 3), (33, 64, 17), (1, 4, 1)])
+def test_linear_parity(n, k, m):
+    rng = np.random.default_rng(n + k + m)
+    x = rng.integers(0, 256, size=(n, k)).astype(np.uint8)
+    w = rng.integers(-128, 128, size=(m, k)).astype(np.int8)
+    b = rng.integers(-4096, 4097, size=m).astype(np.int32)
+    for bias in (b, None):
+        got = qnn.linear(to_dev(x), to_dev(w), None if bias is None else to_dev(bias))
+        np.testing.assert_array_equal(got.cpu().numpy(), oracle.linear(x, w, bias))
+
+
+@pytest.mark.parametrize("bits", [8, 4, 2])
+@pytest.mark.parametrize("signed", [False, True])
+def test_pack_unpack_parity(bits, signed):
+    allbytes = np.arange(256, dtype=np.uint8)
+    per = 8 // bits
+    vals = oracle.unpack(allbytes, 256 * per, bits, signed)
+    got = qnn.unpack_subbyte(to_dev(allbytes), bits, signed)
+    np.testing.assert_array_equal(got.cpu().numpy().astype(np.int32) if signed or bits < 8 else
+                                  got.cpu().numpy().view(np.uint8), vals)
+    if bits < 8:
+        rng = np.random.default_rng(bits)
+        lo, hi = (-(1 << (bits - 1)), 1 << (bits - 1)) if signed else (0, 1 << bits)
+        v = rng.integers(lo, hi, size=4096)
+        np.testing.assert_array_equal(qnn.pack_subbyte(to_dev(v.astype(np.int8)), bits).cpu().numpy(),
+                                      oracle.pack(v, bits))
+
+
+def test_device_status_clean():
+    qnn.device_status()
