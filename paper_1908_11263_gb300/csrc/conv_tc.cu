@@ -7,7 +7,7 @@
 //
 // GEMM view: rows = 128 consecutive output pixels of one image (MMA M = 128),
 // columns = output channels (MMA N = NT), K = kh * kw * c (tap-major, channel
-// minor: the im2col order of Eq. 6).
+// minor: the im2col order of Eq. 6).  Stride 1.
 //
 // Exactness on fp16 tensor cores.  GB300 has no integer tcgen05 MMA, so the
 // integers are embedded exactly in fp16 and multiplied with fp32 accumulation
@@ -22,23 +22,34 @@
 //     minus 0x4B400000 is the chunk's integer sum.  Longer K is split into
 //     several chunks, summed as integers in the epilogue.
 //   * The offsets are removed exactly with a per-channel constant (128 * sum(W)
-//     or -1024 * sum(W)) folded into the bias by the prep kernel.
+//     or -1024 * sum(W)) folded in by the prep kernel.
 //
 // im2col without copies.  For stride 1, the A operand of tap (i, j) is the
-// staged input shifted by i rows and j columns.  The stage keeps one copy of the
-// input window per horizontal tap j (with zero padding applied), stored as
-// [copy j][8-channel chunk][position][8 x fp16].  Rows of A are then 16 bytes
-// apart for every tap, so the tap (i, j) operand is the same no-swizzle K-major
-// layout started i * ow positions later: one shared-memory descriptor per MMA,
-// no im2col buffer.
+// staged input shifted by i rows and j columns.  The stage keeps one copy of
+// the input window per horizontal tap j (padding columns pre-filled with the
+// encoded zero), stored as [copy j][8-channel chunk][position][8 x fp16].  Rows
+// of A are then 16 bytes apart for every tap, so the tap (i, j) operand is the
+// same no-swizzle K-major layout started i * ow positions later: one
+// shared-memory descriptor per MMA, no im2col buffer.  Descriptor offsets of
+// every (tap, k-step) are tabulated once per CTA, so issuing an MMA costs a
+// table load and two additions.
 //
-// Warp roles (one persistent CTA per SM, 9 warps):
-//   warps 0-3  stage the input window (global u8 -> fp16 in shared memory)
+// Data movement per tile: one bulk (TMA) copy brings the tile's input rows
+// (all channels, HBM -> shared memory); converter warps turn each element
+// into fp16 once and store it into the kw copies; the filters are either
+// resident in shared memory or streamed per (channel slab, tap) by bulk
+// copies.  Accumulators form a ring of up to four TMEM buffers, so the MMAs of
+// the next tile run while the epilogue compresses the current one.
+//
+// Warp roles (one persistent CTA per SM, 11 warps):
+//   warps 0-3  converters: raw u8 window -> fp16 copies
 //   warps 4-7  epilogue: TMEM -> registers, integer sum of chunks, compression,
-//              Q-bit packing, store; they also re-arm the accumulators
-//   warp 8     one thread issues tcgen05.mma and the bulk copy of the filters
+//              Q-bit packing, store
+//   warp 8     MMA issue (the warp runs converged; lane 0 issues tcgen05.mma)
+//   warp 9     bulk copies of input rows (lane 0 issues)
+//   warp 10    bulk copies of filters (lane 0 issues)
 // Every wait is bounded; on a timeout the kernel records QNN_ETIMEOUT in the
-// status word, stops its work, lets its tensor-core work drain and frees TMEM.
+// status word, stops its work, lets its copies and MMAs drain and frees TMEM.
 #include <cuda_fp16.h>
 
 #include <algorithm>
@@ -51,46 +62,86 @@ namespace qnn {
 namespace {
 
 constexpr int kTileM = 128;
-constexpr int kThreads = 9 * 32;
-constexpr int kMmaWarp = 8;
+constexpr int kWarps = 11;
+constexpr int kThreads = kWarps * 32;
+constexpr int kMmaWarp = 8, kRawWarp = 9, kBWarp = 10;
 constexpr uint32_t kMagic = 0x4B400000u;  // bits of 1.5 * 2^23
 constexpr int kMaxSmem = 232448;          // 227 KB opt-in dynamic shared memory per block
+constexpr uint32_t kCopyChunk = 32768;    // bytes per bulk copy instruction
+constexpr int kMaxAccBufs = 4;
+constexpr int kMaxTaps = 64;  // kh * kw limit of the tensor-core kernel
+
+// Per-channel compression constants (two records per channel, see the prep kernel).
+//   rec0 = {lam2, kappa, shift, mode}   rec1 = {beta, ulo, uhi, lambda}
+enum { kModeWide = 0, kModeClamp = 1, kModeDirect = 2 };
 
 struct TcArgs {
     const uint8_t *x;
     uint8_t *y;
-    const uint16_t *wpack;  // [n_ntiles][k_pad/8][nt][8] fp16
-    const int4 *chan;       // [n_ntiles * nt] {beta, kappa, lambda, shift}
+    const uint8_t *wpack;  // fp16 filters [n_ntiles][k_pad/8][nt][8]
+    const int4 *chan;      // [2][n_ntiles * nt] compression records
     int n, h, w, c, m, kh, kw, ph, pw, oh, ow;
-    int c_pad, cs, nslab;
+    int c_pad, cs, nslab, log2_groups;
     int n_ntiles, tiles_per_img;
-    long long total_tiles;
-    int p_alloc, stages;
-    int mmas_per_tile, chunk_mmas, nchunks;
-    unsigned long long ow_inv;  // ceil(2^32 / ow)
-    uint32_t b_bytes, copy_bytes, stage_bytes, tmem_cols;
-    uint32_t off_stages, off_chan, off_bar;
-    int *status;  // device status word
+    int total_tiles;
+    int rows_max, p_alloc;
+    int stages, raw_stages, b_stages, b_resident;
+    int mmas_per_tile, chunk_mmas, nchunks, nbuf;
+    uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, chunk_stride;
+    uint32_t off_raw, off_stages, off_chan, off_tab, off_bar;
+    uint32_t tmem_cols;
+    int *status;
+    uint32_t tap_a16[kMaxTaps];  // per tap (i, j): A offset j*copy + i*ow positions, in 16-byte units
 };
 
-struct Tile {
+// Geometry of one tile: 128 consecutive output pixels of image `img`.
+struct TileGeo {
     int nt, img, ti;
+    int oy_a;   // first output row touched
+    int d0;     // column of the first pixel within that row
+    int rows;   // staged input rows (window height)
+    int r_lo;   // staged rows [r_lo, r_hi) lie inside the image
+    int r_hi;
 };
 
-__device__ __forceinline__ Tile decode_tile(const TcArgs &a, long long t)
+__device__ __forceinline__ TileGeo tile_geo(const TcArgs &a, int t)
 {
-    long long per_nt = static_cast<long long>(a.n) * a.tiles_per_img;
-    Tile r;
-    r.nt = static_cast<int>(t / per_nt);
-    long long rem = t - r.nt * per_nt;
-    r.img = static_cast<int>(rem / a.tiles_per_img);
-    r.ti = static_cast<int>(rem - static_cast<long long>(r.img) * a.tiles_per_img);
-    return r;
+    const int per_nt = a.n * a.tiles_per_img;  // total tiles < 2^31 (checked by the planner)
+    TileGeo g;
+    g.nt = t / per_nt;
+    const int rem = t - g.nt * per_nt;
+    g.img = rem / a.tiles_per_img;
+    g.ti = rem - g.img * a.tiles_per_img;
+    const int p0 = g.ti * kTileM;
+    g.oy_a = p0 / a.ow;
+    g.d0 = p0 - g.oy_a * a.ow;
+    const int out_rows = min((g.d0 + kTileM + a.ow - 1) / a.ow, a.oh - g.oy_a);
+    g.rows = min(a.rows_max, out_rows + a.kh - 1);
+    const int iy0 = g.oy_a - a.ph;
+    g.r_lo = min(g.rows, max(0, -iy0));
+    g.r_hi = max(g.r_lo, min(g.rows, a.h - iy0));
+    return g;
 }
 
-__device__ __forceinline__ uint32_t div_ow(const TcArgs &a, uint32_t q)
+__device__ __forceinline__ int tile_nt(const TcArgs &a, int t) { return t / (a.n * a.tiles_per_img); }
+
+__device__ __forceinline__ bool nt_run_starts(const TcArgs &a, int t)
 {
-    return static_cast<uint32_t>((static_cast<unsigned long long>(q) * a.ow_inv) >> 32);
+    return t == static_cast<int>(blockIdx.x) || tile_nt(a, t - gridDim.x) != tile_nt(a, t);
+}
+
+__device__ __forceinline__ bool nt_run_ends(const TcArgs &a, int t)
+{
+    const int nx = t + gridDim.x;
+    return nx >= a.total_tiles || tile_nt(a, nx) != tile_nt(a, t);
+}
+
+// Warp-converged bounded wait: lane 0 polls, the whole warp gets the result.
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, int *status)
+{
+    int ok = 1;
+    if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, status) ? 1 : 0;
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
 }
 
 // ---------------------------------------------------------------- u8 / sub-byte -> fp16 (8 channels)
@@ -109,7 +160,7 @@ __device__ __forceinline__ uint32_t hsub2(uint32_t a, uint32_t b)
     return d;
 }
 
-// Fill value for positions outside the image (activation 0 in the staged encoding).
+// Encoded activation 0 (padding and channels beyond c).
 template <int BITS>
 __device__ __forceinline__ uint32_t pad_half2()
 {
@@ -153,22 +204,19 @@ __device__ __forceinline__ uint4 cvt_u2x8(uint32_t v16)
     return r;
 }
 
-// Generic (any channel count) conversion of channels c0..c0+7 of one pixel.
+// Any channel count: channels c0.. of the pixel whose packed data starts at element e0 of `src`.
 template <int BITS>
-__device__ __forceinline__ uint4 cvt_generic(const uint8_t *xpix_elem0, long long e0, int c0, int c)
+__device__ __noinline__ uint4 cvt_generic(const uint8_t *src, int e0, int c0, int c)
 {
-    const int slot_ch8[8] = {0, 1, 2, 3, 4, 5, 6, 7};
-    const int slot_chs[8] = {0, 4, 1, 5, 2, 6, 3, 7};
     uint16_t hv[8];
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
-        const int ch = c0 + (BITS == 8 ? slot_ch8[s] : slot_chs[s]);
+        const int ch = c0 + (BITS == 8 ? s : ((s & 1) ? 4 + (s >> 1) : (s >> 1)));
         int v = 0;
         if (ch < c) {
-            const long long e = e0 + ch;
-            const int per = 8 / BITS;
-            const uint8_t byte = __ldg(xpix_elem0 + e / per);
-            v = (byte >> ((e % per) * BITS)) & ((1 << BITS) - 1);
+            const int e = e0 + ch;
+            constexpr int per = 8 / BITS;
+            v = (src[e / per] >> ((e % per) * BITS)) & ((1 << BITS) - 1);
         }
         v += (BITS == 8) ? -128 : 1024;
         hv[s] = __half_as_ushort(__int2half_rn(v));
@@ -183,246 +231,487 @@ __device__ __forceinline__ uint4 cvt_generic(const uint8_t *xpix_elem0, long lon
 
 __device__ __forceinline__ void sts128(uint32_t addr, uint4 v)
 {
-    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-                 : "memory");
+    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w));
 }
 
-// ---------------------------------------------------------------- roles
+// ---------------------------------------------------------------- converters (warps 0-3)
 
-// Warps 0-3: stage the input window of one (tile, channel slab).
+// Rows of the window that lie outside the image read as activation 0.
 template <int BITS>
-__device__ void stage_fill(const TcArgs &a, uint32_t stage_base, int img, int oy_a, int p_used, int slab,
-                           bool vec_ok)
+__device__ __noinline__ void zero_rows(uint32_t stage, int r_lo, int r_hi, int rows, int ow, int kw, int lg,
+                                       uint32_t copy_bytes, uint32_t chunk_stride)
 {
-    const int tid = threadIdx.x;  // 0..127
-    const int groups = a.cs / 8;
+    const int groups = 1 << lg;
     const uint32_t padv = pad_half2<BITS>();
     const uint4 pad4 = make_uint4(padv, padv, padv, padv);
-    const long long img_elem0 = static_cast<long long>(img) * a.h * a.w * a.c;
-    for (int j = 0; j < a.kw; ++j) {
-        for (int g = 0; g < groups; ++g) {
-            const int c0 = slab * a.cs + g * 8;
-            const uint32_t base = stage_base + j * a.copy_bytes + g * a.p_alloc * 16;
-            for (int q = tid; q < p_used; q += 128) {
-                const int r = static_cast<int>(div_ow(a, q));
-                const int ox = q - r * a.ow;
-                const int iy = oy_a - a.ph + r;
-                const int ix = ox + j - a.pw;
-                uint4 v = pad4;
-                if (iy >= 0 && iy < a.h && ix >= 0 && ix < a.w && c0 < a.c) {
-                    const long long e0 = img_elem0 + (static_cast<long long>(iy) * a.w + ix) * a.c;
-                    if (vec_ok) {
-                        const long long byte0 = (e0 + c0) * BITS / 8;
-                        if (BITS == 8) {
-                            v = cvt_u8x8(__ldg(reinterpret_cast<const uint2 *>(a.x + byte0)));
-                        } else if (BITS == 4) {
-                            v = cvt_u4x8(__ldg(reinterpret_cast<const uint32_t *>(a.x + byte0)));
-                        } else {
-                            v = cvt_u2x8(__ldg(reinterpret_cast<const uint16_t *>(a.x + byte0)));
-                        }
-                    } else {
-                        v = cvt_generic<BITS>(a.x, e0, c0, a.c);
-                    }
-                }
-                sts128(base + q * 16, v);
-            }
-        }
+    const int zrows = r_lo + (rows - r_hi);
+    const int per_row = ow * groups * kw;
+    for (int it = threadIdx.x; it < zrows * per_row; it += 128) {
+        const int zr = it / per_row;
+        const int rem = it - zr * per_row;
+        const int r = zr < r_lo ? zr : r_hi + (zr - r_lo);
+        const int ox = rem % ow;
+        const int rest = rem / ow;
+        const int gq = rest & (groups - 1);
+        const int j = rest >> lg;
+        sts128(stage + j * copy_bytes + gq * chunk_stride + (r * ow + ox) * 16, pad4);
     }
 }
 
+// One (tile, channel slab): raw rows in shared memory -> kw fp16 copies.  Each
+// warp takes whole input rows; within a row, eight consecutive lanes handle
+// eight consecutive pixels of one 8-channel group, so every 128-bit store
+// phase writes 128 contiguous bytes and no division by the width is needed.
 template <int BITS>
-__device__ void producer_role(const TcArgs &a, uint8_t *smem, uint64_t *a_full, uint64_t *a_empty)
+__device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *raw, uint8_t *smem_out, uint32_t stage,
+                                              const TileGeo &g, int slab, bool vec)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int lg = a.log2_groups;
+    const int groups = 1 << lg;
+    const int cb = a.c * BITS / 8;  // packed bytes per pixel
+    const int w = a.w, c = a.c, ow = a.ow, pw = a.pw, kw = a.kw, cs = a.cs;
+    const uint32_t row_bytes = a.row_bytes, chunk_stride = a.chunk_stride, jstep = a.copy_bytes - 16;
+    const int row_items = ((w + 7) >> 3) << (3 + lg);
+    const uint32_t padv = pad_half2<BITS>();
+    const uint4 pad4 = make_uint4(padv, padv, padv, padv);
+    for (int r = g.r_lo + warp; r < g.r_hi; r += 4) {
+        const uint8_t *raw_row = raw + (r - g.r_lo) * row_bytes;
+        const uint32_t out_row = stage + r * ow * 16;  // byte offset within the stage area
+        for (int base = lane; base < row_items; base += 64) {
+            int ix[2], gg[2];
+            uint2 rv[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {  // both loads first
+                const int it = base + u * 32;
+                gg[u] = (it >> 3) & (groups - 1);
+                ix[u] = ((it >> (3 + lg)) << 3) + (it & 7);
+                rv[u] = make_uint2(0, 0);
+                const int c0 = slab * cs + gg[u] * 8;
+                if (it < row_items && ix[u] < w && vec && c0 < c) {
+                    const uint8_t *p = raw_row + ix[u] * cb + c0 * BITS / 8;
+                    if (BITS == 8) rv[u] = *reinterpret_cast<const uint2 *>(p);
+                    else if (BITS == 4) rv[u].x = *reinterpret_cast<const uint32_t *>(p);
+                    else rv[u].x = *reinterpret_cast<const uint16_t *>(p);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int it = base + u * 32;
+                if (it >= row_items || ix[u] >= w) continue;
+                const int c0 = slab * cs + gg[u] * 8;
+                uint4 v = pad4;
+                if (c0 < c) {
+                    if (!vec) v = cvt_generic<BITS>(raw_row, ix[u] * c, c0, c);
+                    else if (BITS == 8) v = cvt_u8x8(rv[u]);
+                    else if (BITS == 4) v = cvt_u4x8(rv[u].x);
+                    else v = cvt_u2x8(rv[u].x);
+                }
+                // copy j holds this pixel at column ix + pw - j (predicated stores, no branches)
+                uint8_t *dst = smem_out + out_row + gg[u] * chunk_stride + (ix[u] + pw) * 16;
+#pragma unroll
+                for (int j = 0; j < 5; ++j) {
+                    const int ox = ix[u] + pw - j;
+                    if (j < kw && ox >= 0 && ox < ow) *reinterpret_cast<uint4 *>(dst + j * jstep) = v;
+                }
+                for (int j = 5; j < kw; ++j) {
+                    const int ox = ix[u] + pw - j;
+                    if (ox >= 0 && ox < ow) *reinterpret_cast<uint4 *>(dst + j * jstep) = v;
+                }
+            }
+        }
+    }
+    if (g.r_lo > 0 || g.rows > g.r_hi)
+        zero_rows<BITS>(smem_addr(smem_out) + stage, g.r_lo, g.r_hi, g.rows, a.ow, a.kw, a.log2_groups, a.copy_bytes,
+                        a.chunk_stride);
+}
+
+template <int BITS>
+__device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
+                               uint64_t *a_full, uint64_t *a_empty)
 {
     const uint32_t stages_base = smem_addr(smem + a.off_stages);
-    const bool vec_ok = (a.c % 8) == 0;
-    int stage = 0;
-    uint32_t phase = 0;
-    for (long long t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
-        const Tile tl = decode_tile(a, t);
-        const int p0 = tl.ti * kTileM;
-        const int oy_a = p0 / a.ow;
-        const int d0 = p0 - oy_a * a.ow;
-        const int p_used = min(a.p_alloc, (d0 + kTileM + (a.kh - 1) * a.ow + 7) & ~7);
+    const bool vec = (a.c % 8) == 0;
+    // encoded zero everywhere once: padding columns are never written afterwards
+    {
+        const uint32_t padv = pad_half2<BITS>();
+        const uint4 pad4 = make_uint4(padv, padv, padv, padv);
+        const uint32_t total = a.stages * a.stage_bytes / 16;
+        for (uint32_t i = threadIdx.x; i < total; i += 128) sts128(stages_base + i * 16, pad4);
+    }
+    int rs = 0, stage = 0;
+    uint32_t r_ph = 0, a_ph = 0;
+    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+        const TileGeo g = tile_geo(a, t);
+        if (!warp_wait(&raw_full[rs], r_ph, a.status)) return;
+        const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         for (int slab = 0; slab < a.nslab; ++slab) {
-            if (!mbar_wait(&a_empty[stage], phase ^ 1u, a.status)) return;
-            stage_fill<BITS>(a, stages_base + stage * a.stage_bytes, tl.img, oy_a, p_used, slab, vec_ok);
+            if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
+            convert_stage<BITS>(a, raw, smem + a.off_stages, stage * a.stage_bytes, g, slab, vec);
             fence_proxy_async_smem();
             mbar_arrive(&a_full[stage]);
             if (++stage == a.stages) {
                 stage = 0;
-                phase ^= 1u;
+                a_ph ^= 1u;
             }
+        }
+        mbar_arrive(&raw_empty[rs]);
+        if (++rs == a.raw_stages) {
+            rs = 0;
+            r_ph ^= 1u;
         }
     }
 }
 
-// Warp 8, one thread: filters into shared memory, then the MMA stream.
-__device__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *a_full, uint64_t *a_empty,
-                         uint64_t *acc_full, uint64_t *acc_empty, uint64_t *b_full, uint64_t *done, uint32_t idesc,
-                         int nt_cols)
+// ---------------------------------------------------------------- bulk-copy issuers (warps 9, 10)
+
+// Called by a whole warp; lane 0 arms `bar` with the byte count and issues the copies.
+__device__ __forceinline__ void bulk_copy(uint8_t *dst, const uint8_t *src, uint32_t bytes, uint64_t *bar)
 {
-    const uint32_t b_base = smem_addr(smem);
-    const uint32_t stages_base = smem_addr(smem + a.off_stages);
-    const uint32_t a_lbo = a.p_alloc * 16;
-    const uint32_t b_lbo = nt_cols * 16;
-    int stage = 0;
-    uint32_t a_phase = 0, b_phase = 0, done_phase = 0;
-    uint32_t empty_phase[2] = {0, 0};
-    int buf = 0;
-    int cur_nt = -1;
-    bool ok = true;
-    for (long long t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x) {
-        const Tile tl = decode_tile(a, t);
-        if (tl.nt != cur_nt) {
-            if (cur_nt >= 0) {  // previous filters still in use: drain the tensor core first
-                mma_commit(done);
-                if (!mbar_wait(done, done_phase, a.status)) { ok = false; break; }
-                done_phase ^= 1u;
-            }
-            const uint8_t *src = reinterpret_cast<const uint8_t *>(a.wpack) + static_cast<size_t>(tl.nt) * a.b_bytes;
-            mbar_arrive_expect_tx(b_full, a.b_bytes);
-            for (uint32_t off = 0; off < a.b_bytes; off += 65536u)
-                bulk_g2s(smem + off, src + off, min(65536u, a.b_bytes - off), b_full);
-            if (!mbar_wait(b_full, b_phase, a.status)) { ok = false; break; }
-            b_phase ^= 1u;
-            cur_nt = tl.nt;
+    if ((threadIdx.x & 31) == 0) {
+        mbar_arrive_expect_tx(bar, bytes);
+        for (uint32_t off = 0; off < bytes; off += kCopyChunk)
+            bulk_g2s(dst + off, src + off, min(kCopyChunk, bytes - off), bar);
+    }
+    __syncwarp();
+}
+
+// Steps back over the last `count` armed phases of a ring and waits for each
+// (their copies must land before the block exits).
+__device__ __forceinline__ void drain_ring(uint64_t *full, int slot, uint32_t ph, int nslots, int count, int *status)
+{
+    for (int k = 0; k < nslots && k < count; ++k) {
+        if (--slot < 0) {
+            slot = nslots - 1;
+            ph ^= 1u;
         }
-        const int p0 = tl.ti * kTileM;
-        const int oy_a = p0 / a.ow;
-        const int d0 = p0 - oy_a * a.ow;
-        int in_chunk = 0;
-        int done_mmas = 0;
+        warp_wait(&full[slot], ph, status);
+    }
+}
+
+// Input rows of each tile (all channels, only rows inside the image).
+__device__ __forceinline__ void raw_loader_role(const TcArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty)
+{
+    int rs = 0;
+    uint32_t ph = 0;
+    int issued = 0;
+    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+        const TileGeo g = tile_geo(a, t);
+        if (!warp_wait(&raw_empty[rs], ph ^ 1u, a.status)) break;
+        const uint32_t bytes = (g.r_hi - g.r_lo) * a.row_bytes;
+        if (bytes) {
+            const uint8_t *src =
+                a.x + (static_cast<long long>(g.img) * a.h + (g.oy_a - a.ph + g.r_lo)) * a.row_bytes;
+            bulk_copy(smem + a.off_raw + rs * a.raw_bytes, src, bytes, &raw_full[rs]);
+        } else if ((threadIdx.x & 31) == 0) {
+            mbar_arrive(&raw_full[rs]);
+        }
+        ++issued;
+        if (++rs == a.raw_stages) {
+            rs = 0;
+            ph ^= 1u;
+        }
+    }
+    drain_ring(raw_full, rs, ph, a.raw_stages, issued, a.status);
+}
+
+// Filters: the whole set once per run of tiles with the same output-channel
+// tile (resident), or one [nt x cs] tile per (slab, tap) step (streamed).
+__device__ __forceinline__ void b_loader_role(const TcArgs &a, uint8_t *smem, uint64_t *b_full, uint64_t *b_empty, int nt_cols)
+{
+    int bs = 0;
+    uint32_t ph = 0;
+    int issued = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x) {
+        const int nt = tile_nt(a, t);
+        const uint8_t *wsrc = a.wpack + static_cast<size_t>(nt) * a.b_bytes;
+        if (a.b_resident) {
+            if (!nt_run_starts(a, t)) continue;
+            if (!warp_wait(&b_empty[0], ph ^ 1u, a.status)) break;
+            bulk_copy(smem, wsrc, a.b_bytes, &b_full[0]);
+            ph ^= 1u;
+            ++issued;
+            continue;
+        }
         for (int slab = 0; slab < a.nslab && ok; ++slab) {
-            if (!mbar_wait(&a_full[stage], a_phase, a.status)) { ok = false; break; }
+            for (int tap = 0; tap < a.kh * a.kw; ++tap) {
+                if (!warp_wait(&b_empty[bs], ph ^ 1u, a.status)) {
+                    ok = false;
+                    break;
+                }
+                const int kchunk = (tap * a.c_pad + slab * a.cs) / 8;
+                bulk_copy(smem + bs * a.b_tile_bytes, wsrc + static_cast<size_t>(kchunk) * nt_cols * 16,
+                          a.b_tile_bytes, &b_full[bs]);
+                ++issued;
+                if (++bs == a.b_stages) {
+                    bs = 0;
+                    ph ^= 1u;
+                }
+            }
+        }
+    }
+    if (a.b_resident) drain_ring(b_full, 0, ph, 1, issued, a.status);
+    else drain_ring(b_full, bs, ph, a.b_stages, issued, a.status);
+}
+
+// ---------------------------------------------------------------- MMA issuer (warp 8)
+
+// Issues the MMAs of taps [t0, t1) of one slab: KSTEPS k-steps (16 channels each)
+// per tap.  Descriptors come from uniform values only (tap offsets live in the
+// kernel's parameter block), and the loop body has no conditionals, so the
+// MMAs go out back to back.
+template <int KSTEPS>
+__device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t a_tmpl, uint64_t b_tmpl,
+                                           uint32_t abase, uint32_t bbase, uint32_t tap_b16, uint32_t a_step,
+                                           uint32_t b_step, int t0, int t1, uint32_t idesc)
+{
+#pragma unroll 4
+    for (int t = t0; t < t1; ++t) {
+        const uint64_t ad = a_tmpl + (abase + a.tap_a16[t]);
+        const uint64_t bd = b_tmpl + (bbase + t * tap_b16);
+#pragma unroll
+        for (int kk = 0; kk < KSTEPS; ++kk) mma_f16_ss(d, ad + kk * a_step, bd + kk * b_step, idesc, 1u);
+    }
+}
+
+__device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *a_full,
+                                         uint64_t *a_empty, uint64_t *b_full, uint64_t *b_empty, uint64_t *acc_full,
+                                         uint64_t *acc_empty, uint64_t *done, uint32_t idesc, int nt_cols)
+{
+    const bool leader = (threadIdx.x & 31) == 0;
+    const uint32_t b_lbo = nt_cols * 16;
+    const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
+    const uint64_t b_tmpl = smem_desc(0, b_lbo, 128);
+    const uint32_t stages16 = smem_addr(smem + a.off_stages) >> 4;
+    const uint32_t b16 = smem_addr(smem) >> 4;
+    const uint32_t stage16 = a.stage_bytes >> 4, btile16 = a.b_tile_bytes >> 4;
+    const uint32_t a_step = 2 * (a.chunk_stride >> 4), b_step = 2 * nt_cols;  // one k-step = two 8-channel chunks
+    const uint32_t slab_b16 = (a.cs / 8) * nt_cols;
+    const int ksteps = a.cs / 16;
+    const bool resident = a.b_resident != 0;
+    // resident filters: tap t of slab s sits at t * c_pad/8 chunks; streamed: each tap has its own tile
+    const uint32_t tap_b16 = resident ? (a.c_pad / 8) * nt_cols : 0;
+    const int chunk_taps = a.chunk_mmas / ksteps, taps = a.kh * a.kw;
+    const int nbuf = a.nbuf, nslab = a.nslab, nstages = a.stages, nbstages = a.b_stages;
+    int *const status = a.status;
+    int stage = 0, bs = 0, gc = 0;
+    uint32_t a_ph = 0, b_ph = 0, empty_ph = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x) {
+        const TileGeo g = tile_geo(a, t);
+        if (resident && nt_run_starts(a, t)) {
+            if (!warp_wait(&b_full[0], b_ph, status)) break;
+            b_ph ^= 1u;
+        }
+        int in_chunk = 0, buf = 0;
+        for (int slab = 0; slab < nslab && ok; ++slab) {
+            if (!warp_wait(&a_full[stage], a_ph, status)) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
-            const uint32_t sbase = stages_base + stage * a.stage_bytes;
-            for (int i = 0; i < a.kh && ok; ++i) {
-                for (int j = 0; j < a.kw && ok; ++j) {
-                    const int tap = i * a.kw + j;
-                    for (int kk = 0; kk < a.cs / 16; ++kk) {
-                        if (in_chunk == 0) {
-                            if (!mbar_wait(&acc_empty[buf], empty_phase[buf], a.status)) { ok = false; break; }
-                            empty_phase[buf] ^= 1u;
-                            tc_fence_after();
-                        }
-                        const uint32_t a_addr =
-                            sbase + j * a.copy_bytes + (kk * 2) * a_lbo + (d0 + i * a.ow) * 16;
-                        const int kchunk = (tap * a.c_pad + slab * a.cs + kk * 16) / 8;
-                        const uint32_t b_addr = b_base + kchunk * b_lbo;
-                        mma_f16_ss(tmem_base + buf * nt_cols, smem_desc(a_addr, a_lbo, 128),
-                                   smem_desc(b_addr, b_lbo, 128), idesc, 1u);
-                        ++done_mmas;
-                        if (++in_chunk == a.chunk_mmas || done_mmas == a.mmas_per_tile) {
-                            mma_commit(&acc_full[buf]);
-                            buf ^= 1;
-                            in_chunk = 0;
-                        }
+            const uint32_t abase = stages16 + stage * stage16 + g.d0;
+            int tap = 0;
+            while (tap < taps) {
+                uint32_t bbase = b16 + slab * slab_b16;
+                int seg = taps - tap;
+                if (!resident) {  // one streamed filter tile per tap
+                    if (!warp_wait(&b_full[bs], b_ph, status)) {
+                        ok = false;
+                        break;
+                    }
+                    bbase = b16 + bs * btile16 - tap * tap_b16;
+                    seg = 1;
+                }
+                if (in_chunk == 0) {
+                    buf = gc % nbuf;
+                    if (!warp_wait(&acc_empty[buf], (empty_ph >> buf) & 1u, status)) {
+                        ok = false;
+                        break;
+                    }
+                    empty_ph ^= 1u << buf;
+                    tc_fence_after();
+                }
+                seg = min(seg, chunk_taps - in_chunk);
+                if (leader) {
+                    const uint32_t d = tmem_base + buf * nt_cols;
+                    if (ksteps == 1)
+                        issue_taps<1>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                    else if (ksteps == 2)
+                        issue_taps<2>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                    else
+                        issue_taps<4>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                }
+                __syncwarp();
+                tap += seg;
+                in_chunk += seg;
+                if (in_chunk == chunk_taps || (slab == nslab - 1 && tap == taps)) {
+                    if (leader) mma_commit(&acc_full[buf]);
+                    ++gc;
+                    in_chunk = 0;
+                }
+                if (!resident) {
+                    if (leader) mma_commit(&b_empty[bs]);
+                    if (++bs == nbstages) {
+                        bs = 0;
+                        b_ph ^= 1u;
                     }
                 }
             }
-            mma_commit(&a_empty[stage]);  // the slab is free once these MMAs have read it
-            if (++stage == a.stages) {
+            if (!ok) break;
+            if (leader) mma_commit(&a_empty[stage]);
+            if (++stage == nstages) {
                 stage = 0;
-                a_phase ^= 1u;
+                a_ph ^= 1u;
             }
         }
+        if (leader && resident && nt_run_ends(a, t)) mma_commit(&b_empty[0]);
     }
-    // let every issued MMA finish before TMEM is released
-    mma_commit(done);
-    mbar_wait(done, done_phase, a.status);
+    // every issued MMA completes before TMEM is released
+    if (leader) mma_commit(done);
+    warp_wait(done, 0, status);
 }
 
-// Warps 4-7: drain accumulators, compress, pack, store.
+// ---------------------------------------------------------------- epilogue (warps 4-7)
+
+// Compression of one integer sum u = acc + bias in 64-bit arithmetic.
+__device__ __noinline__ uint32_t compress64(int32_t u, int32_t kappa, int32_t lambda, int32_t shift, uint32_t top)
+{
+    long long t = static_cast<long long>(u) * kappa + lambda;
+    t >>= shift;
+    return t < 0 ? 0u : (t > static_cast<long long>(top) ? top : static_cast<uint32_t>(t));
+}
+
+// Channels whose constants need more than the direct form: raw chunk sum s ->
+// output, by the clamped 32-bit form or the 64-bit routine.
+__device__ __noinline__ uint32_t compress_slow(uint32_t s, int4 r0, int4 r1, uint32_t top)
+{
+    const int32_t u = static_cast<int32_t>(s + static_cast<uint32_t>(r1.x));
+    if (r0.w == kModeClamp) {
+        const int32_t uc = min(max(u, r1.y), r1.z);
+        const int32_t t = (uc * r0.y + r1.w) >> r0.z;
+        return static_cast<uint32_t>(min(max(t, 0), static_cast<int32_t>(top)));
+    }
+    return compress64(u, r0.y, r1.w, r0.z, top);
+}
+
+// Compression (Sec. III-A) of 16 raw sums of one pixel, Q-bit packing
+// (Sec. IV-A) and store of the channels below m.  Direct channels (the common
+// case) compute clip(((s * kappa + lam2) mod 2^32) >> shift): the prep kernel
+// has proved that (acc + bias) * kappa + lambda stays inside int32 for every
+// accumulator the layer can produce, and folded bias, the staging offset and
+// the accumulator pre-load into lam2, so the wrapped 32-bit value is exact.
+template <int BITS>
+__device__ __forceinline__ void compress_store16(const uint32_t (&s)[16], const int4 *rec0, const int4 *rec1,
+                                                 bool direct, int m_first, int valid, uint8_t *dst)
+{
+    constexpr uint32_t top = (1u << BITS) - 1u;
+    constexpr int kWords = 16 * BITS / 32;
+    uint32_t packed[kWords];
+#pragma unroll
+    for (int wd = 0; wd < kWords; ++wd) packed[wd] = 0;
+    if (direct) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const int4 r0 = rec0[m_first + k];
+            const int32_t t = static_cast<int32_t>(s[k] * static_cast<uint32_t>(r0.y) + static_cast<uint32_t>(r0.x))
+                              >> r0.z;
+            const uint32_t yv = static_cast<uint32_t>(min(max(t, 0), static_cast<int32_t>(top)));
+            packed[(k * BITS) / 32] |= yv << ((k * BITS) % 32);
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const uint32_t yv = compress_slow(s[k], rec0[m_first + k], rec1[m_first + k], top);
+            packed[(k * BITS) / 32] |= yv << ((k * BITS) % 32);
+        }
+    }
+    constexpr int kBytes = 16 * BITS / 8;
+    if (valid >= 16 && (reinterpret_cast<uintptr_t>(dst) % kBytes) == 0) {
+        if (BITS == 8) *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        else if (BITS == 4) *reinterpret_cast<uint2 *>(dst) = make_uint2(packed[0], packed[1]);
+        else *reinterpret_cast<uint32_t *>(dst) = packed[0];
+    } else {
+        const int nbytes = min(valid, 16) * BITS / 8;
+#pragma unroll
+        for (int b = 0; b < kBytes; ++b)
+            if (b < nbytes) dst[b] = static_cast<uint8_t>(packed[b / 4] >> (8 * (b % 4)));
+    }
+}
+
 template <int BITS, int NT>
-__device__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
+__device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
                               uint64_t *acc_empty)
 {
+    // TMEM columns: nbuf fp32 accumulators of NT columns each, then (when K
+    // needs several chunks) NT columns of running integer sums.
     const int quarter = (threadIdx.x >> 5) & 3;
     const int lane = threadIdx.x & 31;
     const int row = quarter * 32 + lane;  // tile row = output pixel within the tile
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16);
-    const int4 *chan = reinterpret_cast<const int4 *>(smem + a.off_chan);
-    const uint32_t top = (1u << BITS) - 1u;
-    const long long pix_per_img = static_cast<long long>(a.oh) * a.ow;
+    const uint32_t sum_addr = lane_addr + a.nbuf * NT;
+    const int mp = a.n_ntiles * NT;
+    const int4 *rec0 = reinterpret_cast<const int4 *>(smem + a.off_chan);
+    const int4 *rec1 = rec0 + mp;
+    const uint8_t *gdirect = reinterpret_cast<const uint8_t *>(rec1 + mp);  // per 16-channel group
+    const int pix_per_img = a.oh * a.ow;
     const int out_row_bytes = a.m * BITS / 8;
+    const int nbuf = a.nbuf, nchunks = a.nchunks, m = a.m;
+    uint8_t *const ybase = a.y;
+    int *const status = a.status;
 
-    // arm both accumulators with the magic value
-#pragma unroll
-    for (int b = 0; b < 2; ++b)
-#pragma unroll
-        for (int col = 0; col < NT; col += 16) tmem_st16_fill(lane_addr + b * NT + col, kMagic);
+    for (int col = 0; col < nbuf * NT; col += 16) tmem_st16_fill(lane_addr + col, kMagic);
     tmem_wait_st();
     tc_fence_before();
-    mbar_arrive(&acc_empty[0]);
-    mbar_arrive(&acc_empty[1]);
+    for (int b = 0; b < nbuf; ++b) mbar_arrive(&acc_empty[b]);
 
-    uint32_t full_phase[2] = {0, 0};
-    int buf = 0;
-    for (long long t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
-        const Tile tl = decode_tile(a, t);
-        uint32_t s[NT];
-        for (int ch = 0; ch < a.nchunks; ++ch) {
-            // warp-uniform bounded wait (lane 0 polls, the warp follows)
-            int okw = 1;
-            if (lane == 0) okw = mbar_wait(&acc_full[buf], full_phase[buf], a.status) ? 1 : 0;
+    uint32_t full_ph = 0;
+    int gc = 0;
+    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+        const TileGeo g = tile_geo(a, t);
+        // Pixels past the end of the image are computed but not stored.  TMEM
+        // accesses are warp-collective, so every lane executes them; only the
+        // store depends on the lane's pixel.
+        const int p = g.ti * kTileM + row;
+        const int m0 = g.nt * NT;
+        const bool pix_ok = p < pix_per_img;
+        uint8_t *dst_row =
+            ybase + (static_cast<long long>(g.img) * pix_per_img + (pix_ok ? p : 0)) * out_row_bytes;
+        for (int ch = 0; ch < nchunks; ++ch) {
+            const int buf = gc % nbuf;
+            int okw = 1;  // warp-uniform bounded wait
+            if (lane == 0) okw = mbar_wait(&acc_full[buf], (full_ph >> buf) & 1u, status) ? 1 : 0;
             okw = __shfl_sync(0xffffffffu, okw, 0);
             if (!okw) return;
-            full_phase[buf] ^= 1u;
+            full_ph ^= 1u << buf;
             tc_fence_after();
-#pragma unroll
+            const uint32_t acc_addr = lane_addr + buf * NT;
+            const bool last = ch == nchunks - 1;
+#pragma unroll 1
             for (int col = 0; col < NT; col += 16) {
-                uint32_t v[16];
-                tmem_ld16(lane_addr + buf * NT + col, v);
+                uint32_t v[16], prev[16];
+                tmem_ld16(acc_addr + col, v);
+                if (ch > 0) tmem_ld16(sum_addr + col, prev);
                 tmem_wait_ld();
+                if (ch > 0) {
 #pragma unroll
-                for (int k = 0; k < 16; ++k) s[col + k] = (ch == 0) ? v[k] : s[col + k] + v[k];
+                    for (int k = 0; k < 16; ++k) v[k] += prev[k];
+                }
+                tmem_st16_fill(acc_addr + col, kMagic);
+                if (!last) {
+                    tmem_st16(sum_addr + col, v);
+                } else {
+                    const int valid = m - (m0 + col);  // same for the whole warp
+                    if (pix_ok && valid > 0)
+                        compress_store16<BITS>(v, rec0, rec1, gdirect[(m0 + col) >> 4] != 0, m0 + col, valid,
+                                               dst_row + (m0 + col) * BITS / 8);
+                }
             }
-#pragma unroll
-            for (int col = 0; col < NT; col += 16) tmem_st16_fill(lane_addr + buf * NT + col, kMagic);
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(&acc_empty[buf]);
-            buf ^= 1;
-        }
-        // compression (Sec. III-A) and Q-bit packing (Sec. IV-A)
-        const long long p = static_cast<long long>(tl.ti) * kTileM + row;
-        const int m0 = tl.nt * NT;
-        const int mv = min(NT, a.m - m0);
-        if (p < pix_per_img && mv > 0) {
-            constexpr int kWords = NT * BITS / 32 > 0 ? NT * BITS / 32 : 1;
-            uint32_t packed[kWords];
-#pragma unroll
-            for (int wd = 0; wd < kWords; ++wd) packed[wd] = 0;
-#pragma unroll
-            for (int k = 0; k < NT; ++k) {
-                const int4 prm = chan[m0 + k];
-                const int32_t u = static_cast<int32_t>(s[k] + static_cast<uint32_t>(prm.x));
-                long long tq = static_cast<long long>(u) * prm.y + prm.z;
-                tq >>= prm.w;
-                const uint32_t yv = tq < 0 ? 0u : (tq > static_cast<long long>(top) ? top : static_cast<uint32_t>(tq));
-                packed[(k * BITS) / 32] |= yv << ((k * BITS) % 32);
-            }
-            uint8_t *dst = a.y + (static_cast<long long>(tl.img) * pix_per_img + p) * out_row_bytes + m0 * BITS / 8;
-            const int nbytes = mv * BITS / 8;
-            const bool v16 = ((reinterpret_cast<uintptr_t>(dst) | nbytes) & 15) == 0;
-            const bool v4 = ((reinterpret_cast<uintptr_t>(dst) | nbytes) & 3) == 0;
-            if (v16) {
-#pragma unroll
-                for (int wd = 0; wd + 4 <= kWords; wd += 4)
-                    if (wd * 4 < nbytes)
-                        *reinterpret_cast<uint4 *>(dst + wd * 4) =
-                            make_uint4(packed[wd], packed[wd + 1], packed[wd + 2], packed[wd + 3]);
-            } else if (v4) {
-#pragma unroll
-                for (int wd = 0; wd < kWords; ++wd)
-                    if (wd * 4 < nbytes) *reinterpret_cast<uint32_t *>(dst + wd * 4) = packed[wd];
-            } else {
-#pragma unroll
-                for (int wd = 0; wd < kWords; ++wd)
-#pragma unroll
-                    for (int bb = 0; bb < 4; ++bb)
-                        if (wd * 4 + bb < nbytes) dst[wd * 4 + bb] = static_cast<uint8_t>(packed[wd] >> (8 * bb));
-            }
+            ++gc;
         }
     }
 }
@@ -432,36 +721,53 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
 {
     extern __shared__ __align__(128) uint8_t smem[];
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + a.off_bar);
-    uint64_t *a_full = bars;
-    uint64_t *a_empty = bars + a.stages;
-    uint64_t *acc_full = bars + 2 * a.stages;
-    uint64_t *acc_empty = acc_full + 2;
-    uint64_t *b_full = acc_empty + 2;
-    uint64_t *done = b_full + 1;
+    uint64_t *raw_full = bars;
+    uint64_t *raw_empty = raw_full + a.raw_stages;
+    uint64_t *a_full = raw_empty + a.raw_stages;
+    uint64_t *a_empty = a_full + a.stages;
+    uint64_t *b_full = a_empty + a.stages;
+    uint64_t *b_empty = b_full + a.b_stages;
+    uint64_t *acc_full = b_empty + a.b_stages;
+    uint64_t *acc_empty = acc_full + kMaxAccBufs;
+    uint64_t *done = acc_empty + kMaxAccBufs;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
     const int warp = threadIdx.x >> 5;
 
     if (warp == kMmaWarp) {
         if ((threadIdx.x & 31) == 0) {
+            for (int s = 0; s < a.raw_stages; ++s) {
+                mbar_init(&raw_full[s], 1);
+                mbar_init(&raw_empty[s], 128);
+            }
             for (int s = 0; s < a.stages; ++s) {
                 mbar_init(&a_full[s], 128);
                 mbar_init(&a_empty[s], 1);
             }
-            for (int b = 0; b < 2; ++b) {
+            for (int s = 0; s < a.b_stages; ++s) {
+                mbar_init(&b_full[s], 1);
+                mbar_init(&b_empty[s], 1);
+            }
+            for (int b = 0; b < kMaxAccBufs; ++b) {
                 mbar_init(&acc_full[b], 1);
                 mbar_init(&acc_empty[b], 128);
             }
-            mbar_init(b_full, 1);
             mbar_init(done, 1);
             fence_mbar_init();
         }
         __syncwarp();
         tmem_alloc(tmem_slot, a.tmem_cols);
         tmem_relinquish();
-    } else if (warp >= 4) {
+    } else if (warp >= 4 && warp < 8) {
+        // compression records, plus one "all direct" flag per 16-channel group
         int4 *chan = reinterpret_cast<int4 *>(smem + a.off_chan);
         const int mp = a.n_ntiles * NT;
-        for (int i = threadIdx.x - 128; i < mp; i += 128) chan[i] = a.chan[i];
+        for (int i = threadIdx.x - 128; i < 2 * mp; i += 128) chan[i] = a.chan[i];
+        uint8_t *gdirect = reinterpret_cast<uint8_t *>(chan + 2 * mp);
+        for (int gi = threadIdx.x - 128; gi < mp / 16; gi += 128) {
+            int all = 1;
+            for (int k = 0; k < 16; ++k) all &= a.chan[gi * 16 + k].w == kModeDirect;
+            gdirect[gi] = static_cast<uint8_t>(all);
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -469,12 +775,16 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     const uint32_t tmem_base = *tmem_slot;
 
     if (warp < 4) {
-        producer_role<BITS>(a, smem, a_full, a_empty);
+        converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
     } else if (warp < 8) {
         epilogue_role<BITS, NT>(a, smem, tmem_base, acc_full, acc_empty);
-    } else if ((threadIdx.x & 31) == 0) {
-        mma_role(a, smem, tmem_base, a_full, a_empty, acc_full, acc_empty, b_full, done,
+    } else if (warp == kMmaWarp) {
+        mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
                  idesc_f16_f32(kTileM, NT), NT);
+    } else if (warp == kRawWarp) {
+        raw_loader_role(a, smem, raw_full, raw_empty);
+    } else if (warp == kBWarp) {
+        b_loader_role(a, smem, b_full, b_empty, NT);
     }
 
     tc_fence_before();
@@ -487,8 +797,49 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
 
 // ---------------------------------------------------------------- filter / constant preparation
 
+__device__ __forceinline__ long long floor_div(long long a, long long b)
+{
+    long long q = a / b;
+    if ((a % b != 0) && ((a < 0) != (b < 0))) --q;
+    return q;
+}
+
+__device__ __forceinline__ long long ceil_div(long long a, long long b) { return -floor_div(-a, b); }
+
+__device__ __forceinline__ bool in_i32(long long v) { return v >= INT32_MIN && v <= INT32_MAX; }
+
+// For y(u) = clip(floor((u*kappa + lambda) / 2^s), 0, top): an interval [ulo, uhi]
+// outside which y is constant (0 or top, whichever side), chosen so that
+// clamping u into it never changes y.  Returns true when u*kappa + lambda stays
+// inside int32 for every u in the interval (the clamped 32-bit form is exact).
+__device__ bool saturation_bounds(long long kappa, long long lambda, int s, long long top, long long *ulo,
+                                  long long *uhi)
+{
+    const long long one = 1ll << s;
+    if (kappa > 0) {
+        *ulo = ceil_div(one - lambda, kappa) - 1;    // y(u) = 0 for every u <= ulo
+        *uhi = ceil_div(top * one - lambda, kappa);  // y(u) = top for every u >= uhi
+    } else if (kappa < 0) {
+        *ulo = floor_div(top * one - lambda, kappa);  // y(u) = top for every u <= ulo
+        *uhi = floor_div(one - lambda, kappa) + 1;    // y(u) = 0 for every u >= uhi
+    } else {
+        *ulo = 0;
+        *uhi = 0;
+    }
+    if (*ulo < INT32_MIN) *ulo = INT32_MIN;
+    if (*uhi > INT32_MAX) *uhi = INT32_MAX;
+    if (*ulo > *uhi) *ulo = *uhi;
+    return in_i32(*ulo * kappa + lambda) && in_i32(*uhi * kappa + lambda);
+}
+
 // One block per (padded) output channel: fp16 filters in the [ntile][k/8][nt][8]
-// layout of the B operand, and the per-channel constants of the epilogue.
+// layout of the B operand, and the channel's compression records:
+//   rec0 = {lam2, kappa, shift, mode}, rec1 = {beta, ulo, uhi, lambda}
+// where the epilogue's raw sum s (sum of the chunks' bit patterns) relates to the
+// accumulator by acc + bias = s + beta (mod 2^32), and lam2 = beta*kappa + lambda
+// (mod 2^32).  Mode "direct" holds when (acc + bias)*kappa + lambda fits int32 for
+// every accumulator this channel's weights can produce (activations in
+// [0, 2^Q-1]); mode "clamp" when the saturation bounds allow a 32-bit form.
 template <int BITS>
 __global__ void __launch_bounds__(128) conv_tc_prep_kernel(const uint8_t *w, const int32_t *bias, const int16_t *kappa,
                                                            const int32_t *lambda, const uint8_t *shifts, int shift,
@@ -498,7 +849,7 @@ __global__ void __launch_bounds__(128) conv_tc_prep_kernel(const uint8_t *w, con
     const int o = blockIdx.x;
     const int tile = o / nt, col = o % nt;
     const int slot_of[8] = {0, 2, 4, 6, 1, 3, 5, 7};  // inverse of {0,4,1,5,2,6,3,7}
-    long long sum = 0;
+    long long sum = 0, pos = 0, neg = 0;
     for (int k = threadIdx.x; k < k_pad; k += blockDim.x) {
         const int tap = k / c_pad, cc = k - tap * c_pad;
         int v = 0;
@@ -513,30 +864,43 @@ __global__ void __launch_bounds__(128) conv_tc_prep_kernel(const uint8_t *w, con
             }
         }
         sum += v;
+        if (v > 0) pos += v;
+        else neg += v;
         const int slot = BITS == 8 ? (cc & 7) : slot_of[cc & 7];
         const size_t dst = ((static_cast<size_t>(tile) * (k_pad / 8) + k / 8) * nt + col) * 8 + slot;
         wpack[dst] = __half_as_ushort(__int2half_rn(v));
     }
-    __shared__ long long red[128];
-    red[threadIdx.x] = sum;
+    __shared__ long long red[3][128];
+    red[0][threadIdx.x] = sum;
+    red[1][threadIdx.x] = pos;
+    red[2][threadIdx.x] = neg;
     __syncthreads();
     for (int s = 64; s > 0; s >>= 1) {
-        if (threadIdx.x < s) red[threadIdx.x] += red[threadIdx.x + s];
+        if (threadIdx.x < s)
+            for (int r = 0; r < 3; ++r) red[r][threadIdx.x] += red[r][threadIdx.x + s];
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        int4 p = make_int4(0, 0, 0, 0);
+        int4 r0 = make_int4(0, 0, 0, kModeDirect), r1 = make_int4(0, 0, 0, 0);
         if (o < m) {
             const long long off = (BITS == 8) ? -128 : 1024;  // staged activation = x + off
-            const uint32_t beta = static_cast<uint32_t>(bias ? bias[o] : 0) -
-                                  static_cast<uint32_t>(off * red[0]) -
+            const int32_t b = bias ? bias[o] : 0;
+            const uint32_t beta = static_cast<uint32_t>(b) - static_cast<uint32_t>(off * red[0][0]) -
                                   static_cast<uint32_t>(nchunks) * kMagic;
-            p.x = static_cast<int32_t>(beta);
-            p.y = kappa[o];
-            p.z = lambda[o];
-            p.w = shifts ? shifts[o] : shift;
+            const int32_t kap = kappa[o], lam = lambda[o], sh = shifts ? shifts[o] : shift;
+            const long long top = (1 << BITS) - 1;
+            // every accumulator of this channel lies in [top * neg, top * pos]
+            const long long u0 = top * red[2][0] + b, u1 = top * red[1][0] + b;
+            const bool direct = in_i32(u0 * kap + lam) && in_i32(u1 * kap + lam);
+            long long ulo, uhi;
+            const bool clamp = saturation_bounds(kap, lam, sh, top, &ulo, &uhi);
+            const int mode = direct ? kModeDirect : clamp ? kModeClamp : kModeWide;
+            const uint32_t lam2 = beta * static_cast<uint32_t>(kap) + static_cast<uint32_t>(lam);
+            r0 = make_int4(static_cast<int32_t>(lam2), kap, sh, mode);
+            r1 = make_int4(static_cast<int32_t>(beta), static_cast<int32_t>(ulo), static_cast<int32_t>(uhi), lam);
         }
-        chan[o] = p;
+        chan[o] = r0;
+        chan[gridDim.x + o] = r1;
     }
 }
 
@@ -575,6 +939,13 @@ cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, 
     }
 }
 
+uint32_t round_up(uint32_t v, uint32_t a) { return (v + a - 1) / a * a; }
+
+size_t chan_offset(const TcPlan &plan)
+{
+    return (static_cast<size_t>(plan.n_ntiles) * plan.b_bytes + 255) / 256 * 256;
+}
+
 }  // namespace
 
 TcPlan plan_conv_tc(const ConvShape &s)
@@ -582,49 +953,93 @@ TcPlan plan_conv_tc(const ConvShape &s)
     TcPlan p{};
     p.ok = false;
     if (s.sh != 1 || s.sw != 1 || s.oh <= 0 || s.ow <= 0) return p;
+    if (s.kh * s.kw > kMaxTaps) return p;
+    const long long row_bytes = static_cast<long long>(s.w) * s.c * s.bits / 8;
+    if (row_bytes % 16 != 0 || row_bytes > (1 << 20)) return p;  // rows move as whole bulk copies
     const int mp16 = (s.m + 15) / 16 * 16;
     p.nt = mp16 <= 16 ? 16 : mp16 <= 32 ? 32 : mp16 <= 64 ? 64 : 128;
     p.n_ntiles = (s.m + p.nt - 1) / p.nt;
     p.c_pad = (s.c + 15) / 16 * 16;
     p.k_pad = s.kh * s.kw * p.c_pad;
-    p.p_alloc = ((s.ow - 1) + kTileM + (s.kh - 1) * s.ow + 7) / 8 * 8;
+    p.row_bytes = static_cast<uint32_t>(row_bytes);
+    const int out_rows = std::min((s.ow - 1 + kTileM + s.ow - 1) / s.ow, s.oh);
+    p.rows_max = out_rows + s.kh - 1;
+    // positions per copy: the staged rows, and at least everything the 128 tile rows can address
+    const int reach = (s.ow - 1) + kTileM + (s.kh - 1) * s.ow;
+    p.p_alloc = static_cast<int>(round_up(static_cast<uint32_t>(std::max(p.rows_max * s.ow, reach)), 8));
     if (p.p_alloc * 16 >= (1 << 18)) return p;  // descriptor offset field
+    p.raw_bytes = round_up(static_cast<uint32_t>(p.rows_max * row_bytes), 128);
+    if (p.raw_bytes >= (1u << 20)) return p;    // single transaction count
     p.b_bytes = static_cast<uint32_t>(p.nt) * p.k_pad * 2;
-    if (p.b_bytes >= (1u << 20)) return p;  // single transaction count
-    p.tmem_cols = 2 * p.nt < 32 ? 32 : 2 * p.nt;
-    const int mp = p.n_ntiles * p.nt;
-    for (int cs : {64, 32, 16}) {
-        if (cs > p.c_pad || p.c_pad % cs) continue;
-        for (int stages : {3, 2}) {
-            const uint32_t copy_bytes = static_cast<uint32_t>(p.p_alloc) * cs * 2;
-            const uint32_t stage_bytes = copy_bytes * s.kw;
-            const uint32_t off_stages = (p.b_bytes + 127) / 128 * 128;
-            const uint32_t off_chan = off_stages + stages * stage_bytes;
-            const uint32_t off_bar = off_chan + mp * 16;
-            const uint32_t total = off_bar + (2 * stages + 6) * 8 + 16;
-            if (total <= static_cast<uint32_t>(kMaxSmem)) {
-                p.cs = cs;
-                p.nslab = p.c_pad / cs;
-                p.stages = stages;
-                p.copy_bytes = copy_bytes;
-                p.stage_bytes = stage_bytes;
-                p.smem_bytes = total;
-                break;
-            }
-        }
-        if (p.cs) break;
-    }
-    if (!p.cs) return p;
-    p.tiles_per_img = static_cast<int>((static_cast<long long>(s.oh) * s.ow + kTileM - 1) / kTileM);
-    p.total_tiles = static_cast<long long>(p.n_ntiles) * s.n * p.tiles_per_img;
     p.mmas_per_tile = p.k_pad / 16;
     // products per exact chunk: |staged x| * |w| <= 2^14 (INT-8), 1039*8 (INT-4), 1027*2 (INT-2)
     const long long max_prod = s.bits == 8 ? 16384 : s.bits == 4 ? 1039 * 8 : 1027 * 2;
-    const int limit = static_cast<int>(((1ll << 22) / max_prod) / 16);
-    p.nchunks = (p.mmas_per_tile + limit - 1) / limit;
-    p.chunk_mmas = (p.mmas_per_tile + p.nchunks - 1) / p.nchunks;
-    p.nchunks = (p.mmas_per_tile + p.chunk_mmas - 1) / p.chunk_mmas;
-    p.workspace_bytes = (static_cast<size_t>(p.n_ntiles) * p.b_bytes + 255) / 256 * 256 + static_cast<size_t>(mp) * 16;
+    const int limit = static_cast<int>(((1ll << 22) / max_prod) / 16);  // MMAs per exact chunk
+    p.limit_mmas = limit;
+    const int mp = p.n_ntiles * p.nt;
+    const uint32_t chan_bytes = round_up(mp * 32 + mp / 16, 16);
+    p.raw_stages = 2;
+    for (int resident = 1; resident >= 0 && !p.cs; --resident) {
+        if (resident && p.b_bytes > 120u * 1024u) continue;
+        for (int cs : {64, 32, 16}) {
+            if (cs > p.c_pad || p.c_pad % cs) continue;
+            const uint32_t tab_bytes = round_up(s.kh * s.kw * (cs / 16) * 8, 16);
+            for (int stages : {3, 2}) {
+                for (int bst : {4, 3, 2}) {
+                    if (resident && bst != 4) continue;
+                    const int b_stages = resident ? 1 : bst;
+                    const uint32_t b_tile = static_cast<uint32_t>(p.nt) * cs * 2;
+                    const uint32_t b_region = resident ? round_up(p.b_bytes, 128) : b_stages * b_tile;
+                    const uint32_t copy_bytes = static_cast<uint32_t>(p.p_alloc) * cs * 2;
+                    const uint32_t stage_bytes = copy_bytes * s.kw;
+                    const uint32_t off_raw = round_up(b_region, 128);
+                    const uint32_t off_stages = off_raw + p.raw_stages * p.raw_bytes;
+                    const uint32_t off_chan = off_stages + stages * stage_bytes;
+                    const uint32_t off_tab = off_chan + chan_bytes;
+                    const uint32_t off_bar = off_tab + tab_bytes;
+                    const uint32_t nbars = 2 * p.raw_stages + 2 * stages + 2 * b_stages + 2 * kMaxAccBufs + 1;
+                    const uint32_t total = off_bar + nbars * 8 + 16;
+                    if (total > static_cast<uint32_t>(kMaxSmem)) continue;
+                    p.cs = cs;
+                    p.nslab = p.c_pad / cs;
+                    p.stages = stages;
+                    p.b_stages = b_stages;
+                    p.b_resident = resident;
+                    p.b_tile_bytes = b_tile;
+                    p.copy_bytes = copy_bytes;
+                    p.stage_bytes = stage_bytes;
+                    p.off_raw = off_raw;
+                    p.off_stages = off_stages;
+                    p.off_chan = off_chan;
+                    p.off_tab = off_tab;
+                    p.off_bar = off_bar;
+                    p.smem_bytes = total;
+                    break;
+                }
+                if (p.cs) break;
+            }
+            if (p.cs) break;
+        }
+    }
+    if (!p.cs) return p;
+    {
+        // chunks hold whole taps (every k-step of a tap goes to one accumulator)
+        const int ksteps = p.cs / 16, units = p.mmas_per_tile / ksteps;
+        const int limit_units = std::max(1, p.limit_mmas / ksteps);
+        int nch = (units + limit_units - 1) / limit_units;
+        const int per = (units + nch - 1) / nch;
+        p.nchunks = (units + per - 1) / per;
+        p.chunk_mmas = per * ksteps;
+    }
+    // accumulator ring: up to four buffers, plus the integer sums when K takes several chunks
+    const int sum_cols = p.nchunks > 1 ? p.nt : 0;
+    p.nbuf = std::min(kMaxAccBufs, (512 - sum_cols) / p.nt);
+    p.tmem_cols = 32;
+    while (p.tmem_cols < static_cast<uint32_t>(p.nbuf * p.nt + sum_cols)) p.tmem_cols *= 2;
+    p.tiles_per_img = static_cast<int>((static_cast<long long>(s.oh) * s.ow + kTileM - 1) / kTileM);
+    p.total_tiles = static_cast<long long>(p.n_ntiles) * s.n * p.tiles_per_img;
+    if (p.total_tiles >= (1ll << 31)) return p;
+    p.workspace_bytes = chan_offset(p) + static_cast<size_t>(mp) * 32;
     p.ok = true;
     return p;
 }
@@ -633,26 +1048,17 @@ cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const Co
                                 cudaStream_t st)
 {
     uint16_t *wpack = static_cast<uint16_t *>(workspace);
-    int4 *chan = reinterpret_cast<int4 *>(static_cast<uint8_t *>(workspace) +
-                                          (static_cast<size_t>(plan.n_ntiles) * plan.b_bytes + 255) / 256 * 256);
+    int4 *chan = reinterpret_cast<int4 *>(static_cast<uint8_t *>(workspace) + chan_offset(plan));
     const int mp = plan.n_ntiles * plan.nt;
+#define QNN_PREP(B)                                                                                               \
+    conv_tc_prep_kernel<B><<<mp, 128, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, s.kh, s.kw, \
+                                               s.c, plan.c_pad, plan.k_pad, plan.nt, plan.nchunks, wpack, chan)
     switch (s.bits) {
-        case 8:
-            conv_tc_prep_kernel<8><<<mp, 128, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, s.kh,
-                                                       s.kw, s.c, plan.c_pad, plan.k_pad, plan.nt, plan.nchunks,
-                                                       wpack, chan);
-            break;
-        case 4:
-            conv_tc_prep_kernel<4><<<mp, 128, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, s.kh,
-                                                       s.kw, s.c, plan.c_pad, plan.k_pad, plan.nt, plan.nchunks,
-                                                       wpack, chan);
-            break;
-        default:
-            conv_tc_prep_kernel<2><<<mp, 128, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, s.kh,
-                                                       s.kw, s.c, plan.c_pad, plan.k_pad, plan.nt, plan.nchunks,
-                                                       wpack, chan);
-            break;
+        case 8: QNN_PREP(8); break;
+        case 4: QNN_PREP(4); break;
+        default: QNN_PREP(2); break;
     }
+#undef QNN_PREP
     return cudaGetLastError();
 }
 
@@ -660,27 +1066,32 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
                                const void *workspace, cudaStream_t st)
 {
     if (s.n == 0) return cudaSuccess;
-    const uint16_t *wpack = static_cast<const uint16_t *>(workspace);
-    const int4 *chan = reinterpret_cast<const int4 *>(static_cast<const uint8_t *>(workspace) +
-                                                      (static_cast<size_t>(plan.n_ntiles) * plan.b_bytes + 255) / 256 * 256);
-    const int mp = plan.n_ntiles * plan.nt;
     TcArgs a{};
     a.x = x;
     a.y = y;
-    a.wpack = wpack;
-    a.chan = chan;
+    a.wpack = static_cast<const uint8_t *>(workspace);
+    a.chan = reinterpret_cast<const int4 *>(static_cast<const uint8_t *>(workspace) + chan_offset(plan));
     a.n = s.n; a.h = s.h; a.w = s.w; a.c = s.c; a.m = s.m; a.kh = s.kh; a.kw = s.kw;
     a.ph = s.ph; a.pw = s.pw; a.oh = s.oh; a.ow = s.ow;
     a.c_pad = plan.c_pad; a.cs = plan.cs; a.nslab = plan.nslab;
-    a.n_ntiles = plan.n_ntiles; a.tiles_per_img = plan.tiles_per_img; a.total_tiles = plan.total_tiles;
-    a.p_alloc = plan.p_alloc; a.stages = plan.stages;
+    a.log2_groups = plan.cs == 64 ? 3 : plan.cs == 32 ? 2 : 1;
+    a.n_ntiles = plan.n_ntiles; a.tiles_per_img = plan.tiles_per_img;
+    a.total_tiles = static_cast<int>(plan.total_tiles);
+    a.rows_max = plan.rows_max; a.p_alloc = plan.p_alloc;
+    a.stages = plan.stages; a.raw_stages = plan.raw_stages; a.b_stages = plan.b_stages;
+    a.b_resident = plan.b_resident;
     a.mmas_per_tile = plan.mmas_per_tile; a.chunk_mmas = plan.chunk_mmas; a.nchunks = plan.nchunks;
-    a.ow_inv = ((1ull << 32) + s.ow - 1) / s.ow;
-    a.b_bytes = plan.b_bytes; a.copy_bytes = plan.copy_bytes; a.stage_bytes = plan.stage_bytes;
+    a.nbuf = plan.nbuf;
+    a.row_bytes = plan.row_bytes; a.raw_bytes = plan.raw_bytes;
+    a.b_bytes = plan.b_bytes; a.b_tile_bytes = plan.b_tile_bytes;
+    a.copy_bytes = plan.copy_bytes; a.stage_bytes = plan.stage_bytes;
+    a.chunk_stride = plan.p_alloc * 16;
+    a.off_raw = plan.off_raw; a.off_stages = plan.off_stages; a.off_chan = plan.off_chan;
+    a.off_tab = plan.off_tab; a.off_bar = plan.off_bar;
     a.tmem_cols = plan.tmem_cols;
-    a.off_stages = (plan.b_bytes + 127) / 128 * 128;
-    a.off_chan = a.off_stages + plan.stages * plan.stage_bytes;
-    a.off_bar = a.off_chan + mp * 16;
+    for (int i = 0; i < s.kh; ++i)
+        for (int j = 0; j < s.kw; ++j)
+            a.tap_a16[i * s.kw + j] = (j * plan.copy_bytes) / 16 + static_cast<uint32_t>(i * s.ow);
     a.status = device_status_ptr();
     if (!a.status) return cudaErrorInvalidSymbol;
     const long long sms = device_sm_count();

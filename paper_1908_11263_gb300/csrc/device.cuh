@@ -10,17 +10,12 @@
 
 namespace qnn {
 
-// A bounded wait gives up after this many nanoseconds of %globaltimer.
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
+// A bounded wait gives up after this many SM clock cycles (about two seconds at
+// GB300 clocks); each mbarrier poll may park the thread for at most
+// kSuspendHintNs, and the hardware wakes it as soon as the phase completes.
+constexpr long long kWaitLimitCycles = 4000000000ll;
+constexpr uint32_t kSuspendHintNs = 1000000u;
 
-__device__ __forceinline__ uint64_t globaltimer()
-{
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-// Records `code` in the library's device status word (first error wins).
 __device__ __forceinline__ void report(int *status, int code) { atomicCAS(status, 0, code); }
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)
@@ -51,12 +46,12 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
-__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
+__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity)
 {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
         : "r"(smem_addr(bar)), "r"(parity)
@@ -64,21 +59,43 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
     return ok != 0;
 }
 
-// Waits for the phase with the given parity to complete.  Returns false (and
-// records QNN_ETIMEOUT in *status) when kWaitLimitNs pass first.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *status)
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer();
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendHintNs)
+        : "memory");
+    return ok != 0;
+}
+
+// Slow path of mbar_wait: polls with the non-blocking test and a short sleep
+// between polls until the phase completes or `limit_cycles` SM cycles pass
+// (then records QNN_ETIMEOUT and returns false).  Out of line so the many wait
+// sites stay small in the instruction cache.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity, int *status, long long limit_cycles)
+{
+    const long long t0 = clock64();
     while (true) {
-#pragma unroll 1
-        for (int i = 0; i < 32; ++i)
-            if (mbar_try_wait(bar, parity)) return true;
-        if (globaltimer() - t0 > kWaitLimitNs) {
+        if (mbar_test(bar, parity)) return true;
+        __nanosleep(32);
+        if (clock64() - t0 > limit_cycles) {
             report(status, QNN_ETIMEOUT);
             return false;
         }
     }
+}
+
+// Waits for the phase with the given parity to complete.  Returns false (and
+// records QNN_ETIMEOUT in *status) when `limit_cycles` SM cycles pass first.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *status,
+                                          long long limit_cycles = kWaitLimitCycles)
+{
+    if (mbar_test(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, status, limit_cycles);
 }
 
 // ------------------------------------------------------------------ bulk copy (TMA, untiled)
@@ -164,6 +181,17 @@ __device__ __forceinline__ void tmem_st16_fill(uint32_t taddr, uint32_t v)
         "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
         "{%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1};" ::"r"(taddr),
         "r"(v)
+        : "memory");
+}
+
+// Writes 16 consecutive columns of this thread's lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
         : "memory");
 }
 

@@ -34,14 +34,21 @@ struct TcPlan {
     int cs;             // channels per staged slab
     int nslab;          // c_pad / cs
     int k_pad;          // kh * kw * c_pad
+    int rows_max;       // input rows staged per tile (upper bound)
     int p_alloc;        // staged positions per horizontal copy
-    int stages;         // staged slabs in flight
+    int stages;         // converted slabs in flight
+    int raw_stages;     // raw input windows in flight
+    int b_stages;       // filter tiles in flight (1 when resident)
+    int b_resident;     // whole filter set kept in shared memory
     int tiles_per_img;  // ceil(oh * ow / 128)
     long long total_tiles;
     int mmas_per_tile;  // MMAs (K = 16 each) per tile
-    int chunk_mmas;     // MMAs per exact fp32 accumulator chunk
+    int limit_mmas;     // most MMAs one exact fp32 accumulator chunk may take
+    int chunk_mmas;     // MMAs per exact fp32 accumulator chunk (whole taps)
     int nchunks;        // chunks per tile
-    uint32_t b_bytes, copy_bytes, stage_bytes, smem_bytes, tmem_cols;
+    int nbuf;           // TMEM accumulator buffers in the ring
+    uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, smem_bytes, tmem_cols;
+    uint32_t off_raw, off_stages, off_chan, off_tab, off_bar;
     size_t workspace_bytes;
 };
 

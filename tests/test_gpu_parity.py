@@ -68,16 +68,18 @@ def test_conv_random_shapes(shape):
     want = conv_oracle(x, wt, bias, kappa, lam, shifts, shift, bits, stride, pad)
     want_scalar = conv_oracle(x, wt, None, kappa, lam, None, shift, bits, stride, pad)
     desc = qnn.conv_desc(n, h, w, c, m, kh, kw, stride, pad, bits, shift)
+    tc = qnn.conv_algo(desc) == qnn.ALGO_TENSORCORE
     for algo in ALGOS:
-        if algo == qnn.ALGO_TENSORCORE and stride != (1, 1):
+        if algo == qnn.ALGO_TENSORCORE and not tc:
             continue
         got = conv_gpu(x, wt, bias, kappa, lam, shifts, shift, bits, stride, pad, algo)
         assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
         got = conv_gpu(x, wt, None, kappa, lam, None, shift, bits, stride, pad, algo)
         assert first_mismatch(got, want_scalar) is None, (algo, "scalar shift, no bias",
                                                           first_mismatch(got, want_scalar))
-    if stride == (1, 1):
-        assert qnn.conv_algo(desc) == qnn.ALGO_TENSORCORE
+    # the tensor-core kernel takes every stride-1 layer whose input rows are whole 16-byte units
+    if stride == (1, 1) and (w * c * bits // 8) % 16 == 0:
+        assert tc
 
 
 @pytest.mark.parametrize("shift", [0, 1, 31, 40, 62])
@@ -91,18 +93,21 @@ def test_conv_shift_extremes(shift):
 
 
 @pytest.mark.parametrize("xval,wval", [(0, -128), (255, 127), (255, -128), (0, 127), (128, -128), (1, -1)])
-@pytest.mark.parametrize("c", [256, 2304, 1152])
-def test_exact_accumulation_at_the_bounds(xval, wval, c):
-    """Constant 1x1 layers drive every accumulator chunk to its extreme; with kappa=1,
-    shift=0 and lambda = 100 - acc every output reads 100 only if acc is exact."""
-    n, h, w, m = 1, 4, 32, 16
+@pytest.mark.parametrize("k,c", [(1, 256), (3, 128), (3, 256)])
+def test_exact_accumulation_at_the_bounds(xval, wval, k, c):
+    """Constant layers without padding drive every accumulator chunk to its extreme
+    (K = 256, 1152, 2304); with kappa=1, shift=0 and lambda = 100 - acc every output
+    reads 100 only if acc is exact."""
+    n, m = 1, 16
+    h, w = (4, 32) if k == 1 else (6, 6)
     x = np.full((n, h, w, c), xval)
-    wt = np.full((m, 1, 1, c), wval)
+    wt = np.full((m, k, k, c), wval)
     wt[1::2] = -wt[1::2] - (1 if wval > 0 else 0)  # mix signs across channels (stay inside int8)
     wt = np.clip(wt, -128, 127)
     acc = (xval * wt.reshape(m, -1).sum(axis=1)).astype(np.int64)
     lam = (100 - acc).astype(np.int32)
     kappa = np.ones(m, np.int16)
+    assert qnn.conv_algo(qnn.conv_desc(n, h, w, c, m, k, k, 1, 0, 8, 0)) == qnn.ALGO_TENSORCORE
     for algo in ALGOS:
         got = conv_gpu(x, wt, None, kappa, lam, None, 0, 8, (1, 1), (0, 0), algo)
         assert np.all(got == 100), (algo, np.unique(got))
