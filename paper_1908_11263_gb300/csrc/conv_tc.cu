@@ -88,7 +88,7 @@ struct TcArgs {
     int stages, raw_stages, b_stages, b_resident;
     int mmas_per_tile, chunk_mmas, nchunks, nbuf;
     uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, chunk_stride;
-    uint32_t off_raw, off_stages, off_chan, off_tab, off_bar;
+    uint32_t off_raw, off_stages, off_chan, off_bar;
     uint32_t tmem_cols;
     int *status;
     uint32_t tap_a16[kMaxTaps];  // per tap (i, j): A offset j*copy + i*ow positions, in 16-byte units
@@ -983,7 +983,6 @@ TcPlan plan_conv_tc(const ConvShape &s)
         if (resident && p.b_bytes > 120u * 1024u) continue;
         for (int cs : {64, 32, 16}) {
             if (cs > p.c_pad || p.c_pad % cs) continue;
-            const uint32_t tab_bytes = round_up(s.kh * s.kw * (cs / 16) * 8, 16);
             for (int stages : {3, 2}) {
                 for (int bst : {4, 3, 2}) {
                     if (resident && bst != 4) continue;
@@ -995,8 +994,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     const uint32_t off_raw = round_up(b_region, 128);
                     const uint32_t off_stages = off_raw + p.raw_stages * p.raw_bytes;
                     const uint32_t off_chan = off_stages + stages * stage_bytes;
-                    const uint32_t off_tab = off_chan + chan_bytes;
-                    const uint32_t off_bar = off_tab + tab_bytes;
+                    const uint32_t off_bar = off_chan + chan_bytes;
                     const uint32_t nbars = 2 * p.raw_stages + 2 * stages + 2 * b_stages + 2 * kMaxAccBufs + 1;
                     const uint32_t total = off_bar + nbars * 8 + 16;
                     if (total > static_cast<uint32_t>(kMaxSmem)) continue;
@@ -1011,7 +1009,6 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     p.off_raw = off_raw;
                     p.off_stages = off_stages;
                     p.off_chan = off_chan;
-                    p.off_tab = off_tab;
                     p.off_bar = off_bar;
                     p.smem_bytes = total;
                     break;
@@ -1087,7 +1084,7 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.copy_bytes = plan.copy_bytes; a.stage_bytes = plan.stage_bytes;
     a.chunk_stride = plan.p_alloc * 16;
     a.off_raw = plan.off_raw; a.off_stages = plan.off_stages; a.off_chan = plan.off_chan;
-    a.off_tab = plan.off_tab; a.off_bar = plan.off_bar;
+    a.off_bar = plan.off_bar;
     a.tmem_cols = plan.tmem_cols;
     for (int i = 0; i < s.kh; ++i)
         for (int j = 0; j < s.kw; ++j)

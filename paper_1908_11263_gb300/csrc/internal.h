@@ -48,7 +48,7 @@ struct TcPlan {
     int nchunks;        // chunks per tile
     int nbuf;           // TMEM accumulator buffers in the ring
     uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, smem_bytes, tmem_cols;
-    uint32_t off_raw, off_stages, off_chan, off_tab, off_bar;
+    uint32_t off_raw, off_stages, off_chan, off_bar;
     size_t workspace_bytes;
 };
 
