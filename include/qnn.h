@@ -45,7 +45,8 @@ typedef enum {
     QNN_EALIGN = 3,        /* a tensor pointer that must be 16-byte aligned is not */
     QNN_ECUDA = 4,         /* a CUDA runtime call or kernel launch failed */
     QNN_ETIMEOUT = 5,      /* a bounded device-side wait gave up (reported by qnn_device_status) */
-    QNN_EWORKSPACE = 6     /* workspace missing or smaller than qconv_hwc_workspace_size() */
+    QNN_EWORKSPACE = 6,    /* workspace missing or smaller than qconv_hwc_workspace_size() */
+    QNN_ESCRATCH = 7       /* qconv_hwc_noalloc(): the layer needs more than QNN_NOALLOC_SCRATCH_BYTES */
 } qnn_status;
 
 /* Convolution algorithm choice (qnn_conv_desc.algo). */
@@ -134,6 +135,45 @@ qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const v
 /* Which kernel qconv_hwc() would run for d: QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE;
  * negative qnn_status on invalid or unsupported descriptors. */
 int32_t qconv_hwc_algo(const qnn_conv_desc *d);
+
+/* Size of the fixed scratch array behind qconv_hwc_noalloc(): 2 MiB. */
+enum { QNN_NOALLOC_SCRATCH_BYTES = 2097152 };
+
+/*
+ * qconv_hwc() without a workspace, for callers that cannot allocate device
+ * memory.  The paper has no counterpart to this entry point; it serves users of
+ * the library.  Typical such callers: a serving runtime that commits all device
+ * memory to its own arenas up front and has none to hand to a library; a
+ * latency-critical loop, where cudaMalloc / cudaFree would synchronise the
+ * device and stall its other streams; a plain C caller with no device
+ * allocator of its own to size, own and free a workspace.
+ *
+ * Arguments and results are those of qconv_hwc() minus the workspace.  The
+ * re-laid-out filters and per-channel constants go to one scratch array of
+ * QNN_NOALLOC_SCRATCH_BYTES compiled into the library's device image, which
+ * every GPU that loads the library holds until the process exits.  The call
+ * allocates nothing: no cudaMalloc, cudaFree or allocating library routine.
+ *
+ *  - Only for descriptors that select the tensor-core kernel (QNN_ALGO_AUTO
+ *    resolving to it, or QNN_ALGO_TENSORCORE), else QNN_EUNSUPPORTED.  The
+ *    CUDA-core kernel needs no scratch: call qconv_hwc() with a NULL workspace.
+ *  - QNN_ESCRATCH, with nothing enqueued, when the layer needs more than
+ *    QNN_NOALLOC_SCRATCH_BYTES; qconv_hwc_workspace_size() gives the need.
+ *  - Set-up on first use: the first call on each device looks up the scratch
+ *    array's device address (cudaGetSymbolAddress, with that device current;
+ *    QNN_ECUDA if that fails), and the first tensor-core launch of each bit
+ *    width and filter tile on a device raises that kernel's shared-memory
+ *    limit.  Make those first calls before any stream capture.
+ *  - Shared state: all calls on a device use the same array, which keeps the
+ *    last call's contents.  Each call rewrites every scratch byte its
+ *    convolution reads before reading it, so nothing has to be cleared between
+ *    calls.  Calls that overlap on the GPU (streams with no ordering between
+ *    them) race on the array and give undefined results; calls queued on one
+ *    stream do not overlap.
+ */
+qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
+                             const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y,
+                             void *stream);
 
 /*
  * Fully connected layer (Sec. IV-A, matrix-vector product split over output

@@ -105,6 +105,32 @@ qnn_status check_workspace(const TcPlan &plan, const void *workspace, size_t byt
     return QNN_OK;
 }
 
+// Scratch of qconv_hwc_noalloc(): part of the library's device image, so that
+// entry point never allocates.  Each device that loads the library holds its own
+// copy until exit.  In host code the name is only a stand-in for the symbol;
+// the device address comes from cudaGetSymbolAddress.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[QNN_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+
+// Device address of g_noalloc_scratch on the current device, looked up on the
+// first call per device (with that device current); nullptr on failure.  The
+// cache is a fixed array, so this allocates no memory on host or device.
+void *noalloc_scratch_ptr()
+{
+    static std::mutex mu;
+    static void *cache[kMaxDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!cache[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+        cache[dev] = p;
+    }
+    return cache[dev];
+}
+
 }  // namespace
 }  // namespace qnn
 
@@ -198,6 +224,32 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
     return from_cuda(launch_conv_direct(s, p, cs));
 }
 
+qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
+                             const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y,
+                             void *stream)
+{
+    ConvShape s;
+    qnn_status st = check_conv(d, &s);
+    if (st != QNN_OK) return st;
+    if (s.n > 0 && (!x || !y)) return QNN_EINVAL;
+    if (!aligned(x, 16) || !aligned(y, 16)) return QNN_EALIGN;
+    TcPlan plan;
+    st = check_params(d, s, w, bias, kappa, lambda, shifts, &plan);
+    if (st != QNN_OK) return st;
+    if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE) return QNN_EUNSUPPORTED;
+    if (plan.workspace_bytes > static_cast<size_t>(QNN_NOALLOC_SCRATCH_BYTES)) return QNN_ESCRATCH;
+    void *scratch = noalloc_scratch_ptr();
+    if (!scratch) return QNN_ECUDA;
+    // the prep kernel rewrites every scratch byte the convolution reads, so the
+    // previous call's contents never reach this one
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
+                 d->shift, static_cast<uint8_t *>(y)};
+    cudaError_t e = launch_conv_tc_prep(plan, s, p, scratch, cs);
+    if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, scratch, cs);
+    return from_cuda(e);
+}
+
 qnn_status qlinear(int32_t n, int32_t k, int32_t m, const uint8_t *x, const int8_t *w, const int32_t *bias,
                    int32_t *y, void *stream)
 {
@@ -258,6 +310,7 @@ const char *qnn_status_string(qnn_status s)
         case QNN_ECUDA: return "CUDA error";
         case QNN_ETIMEOUT: return "device-side wait timed out";
         case QNN_EWORKSPACE: return "workspace missing or too small";
+        case QNN_ESCRATCH: return "layer needs more scratch than the no-allocation entry point's fixed array holds";
         default: return "unknown status";
     }
 }

@@ -20,10 +20,12 @@ import torch
 from . import build as _build
 
 QNN_OK, QNN_EINVAL, QNN_EUNSUPPORTED, QNN_EALIGN, QNN_ECUDA, QNN_ETIMEOUT, QNN_EWORKSPACE = range(7)
+QNN_ESCRATCH = 7
+NOALLOC_SCRATCH_BYTES = 2 << 20  # QNN_NOALLOC_SCRATCH_BYTES
 ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
-            "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version")
+            "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc")
 
 
 class QnnError(RuntimeError):
@@ -68,6 +70,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_run.argtypes = [DP, P, P, P, SZ, P]
         lib.qconv_hwc_run.restype = I32
         lib.qconv_hwc_algo.argtypes = [DP]
+        lib.qconv_hwc_noalloc.argtypes = [DP, P, P, P, P, P, P, P, P]
+        lib.qconv_hwc_noalloc.restype = I32
         lib.qconv_hwc_algo.restype = I32
         lib.qlinear.argtypes = [I32, I32, I32, P, P, P, P, P]
         lib.qlinear.restype = I32
@@ -184,6 +188,46 @@ def conv_hwc(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, strid
     st = load().qconv_hwc(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(bias), _ptr(kappa), _ptr(lam), _ptr(shifts),
                           _ptr(out), _ptr(workspace), ctypes.c_size_t(nbytes), _stream(stream))
     _check(st, "qconv_hwc")
+    return out
+
+
+def conv_hwc_noalloc(x, w, kappa, lam, out, *, bias=None, shifts=None, shift=0, bits=8, stride=1, pad=0,
+                     algo=ALGO_AUTO, stream=None):
+    """conv_hwc() through qconv_hwc_noalloc(): no device memory is allocated,
+    neither by the library nor here (the caller passes `out`).
+
+    For callers that cannot allocate device memory: a runtime whose memory is
+    all committed to its own arenas, a latency-critical loop where an allocation
+    or free would synchronise the device, a caller with no allocator to own a
+    workspace.  The layer's scratch goes to the library's fixed array of
+    NOALLOC_SCRATCH_BYTES per device; larger layers raise QnnError with status
+    QNN_ESCRATCH.  Only descriptors that select the tensor-core kernel.  The
+    first call on a device does set-up (the array's device address, the
+    kernel's shared-memory limit): make it before any stream capture.  All calls
+    share the array: calls on different streams must not overlap on the GPU.
+    """
+    _dev(x, torch.uint8, "x")
+    _dev(w, (torch.int8, torch.uint8), "w")
+    _dev(kappa, torch.int16, "kappa")
+    _dev(lam, torch.int32, "lambda")
+    _dev(out, torch.uint8, "out")
+    if bias is not None:
+        _dev(bias, torch.int32, "bias")
+    if shifts is not None:
+        _dev(shifts, torch.uint8, "shifts")
+    per = 8 // bits
+    n, h, wd, cb = x.shape
+    m, kh, kw, cb2 = w.shape
+    if cb != cb2:
+        raise ValueError("x and w disagree on the channel count")
+    desc = conv_desc(n, h, wd, cb * per, m, kh, kw, stride, pad, bits, shift, algo)
+    oh = (h + 2 * desc.pad_h - kh) // desc.stride_h + 1
+    ow = (wd + 2 * desc.pad_w - kw) // desc.stride_w + 1
+    if tuple(out.shape) != (n, oh, ow, m // per):
+        raise ValueError(f"out must have shape {(n, oh, ow, m // per)}, got {tuple(out.shape)}")
+    st = load().qconv_hwc_noalloc(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(bias), _ptr(kappa), _ptr(lam),
+                                  _ptr(shifts), _ptr(out), _stream(stream))
+    _check(st, "qconv_hwc_noalloc")
     return out
 
 
