@@ -136,12 +136,10 @@ __device__ __forceinline__ bool nt_run_ends(const TcArgs &a, int t)
     return nx >= a.total_tiles || tile_nt(a, nx) != tile_nt(a, t);
 }
 
-// Warp-converged bounded wait: lane 0 polls, the whole warp gets the result.
+// Warp-converged bounded wait (all lanes poll; the result is warp-uniform).
 __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, int *status)
 {
-    int ok = 1;
-    if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, status) ? 1 : 0;
-    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+    return mbar_wait_warp(bar, parity, status);
 }
 
 // ---------------------------------------------------------------- u8 / sub-byte -> fp16 (8 channels)
@@ -458,9 +456,10 @@ __device__ __forceinline__ void b_loader_role(const TcArgs &a, uint8_t *smem, ui
 // ---------------------------------------------------------------- MMA issuer (warp 8)
 
 // Issues the MMAs of taps [t0, t1) of one slab: KSTEPS k-steps (16 channels each)
-// per tap.  Descriptors come from uniform values only (tap offsets live in the
-// kernel's parameter block), and the loop body has no conditionals, so the
-// MMAs go out back to back.
+// per tap.  Called by the whole converged MMA warp (one elected lane issues).
+// Descriptors come from uniform values only (tap offsets live in the kernel's
+// parameter block), and the loop body has no conditionals, so the MMAs go out
+// back to back.
 template <int KSTEPS>
 __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t a_tmpl, uint64_t b_tmpl,
                                            uint32_t abase, uint32_t bbase, uint32_t tap_b16, uint32_t a_step,
@@ -471,7 +470,7 @@ __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t
         const uint64_t ad = a_tmpl + (abase + a.tap_a16[t]);
         const uint64_t bd = b_tmpl + (bbase + t * tap_b16);
 #pragma unroll
-        for (int kk = 0; kk < KSTEPS; ++kk) mma_f16_ss(d, ad + kk * a_step, bd + kk * b_step, idesc, 1u);
+        for (int kk = 0; kk < KSTEPS; ++kk) mma_f16_ss_warp(d, ad + kk * a_step, bd + kk * b_step, idesc, 1u);
     }
 }
 
@@ -479,7 +478,6 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                                          uint64_t *a_empty, uint64_t *b_full, uint64_t *b_empty, uint64_t *acc_full,
                                          uint64_t *acc_empty, uint64_t *done, uint32_t idesc, int nt_cols)
 {
-    const bool leader = (threadIdx.x & 31) == 0;
     const uint32_t b_lbo = nt_cols * 16;
     const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
     const uint64_t b_tmpl = smem_desc(0, b_lbo, 128);
@@ -534,25 +532,22 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                     tc_fence_after();
                 }
                 seg = min(seg, chunk_taps - in_chunk);
-                if (leader) {
-                    const uint32_t d = tmem_base + buf * nt_cols;
-                    if (ksteps == 1)
-                        issue_taps<1>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
-                    else if (ksteps == 2)
-                        issue_taps<2>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
-                    else
-                        issue_taps<4>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
-                }
-                __syncwarp();
+                const uint32_t d = tmem_base + buf * nt_cols;
+                if (ksteps == 1)
+                    issue_taps<1>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                else if (ksteps == 2)
+                    issue_taps<2>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                else
+                    issue_taps<4>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
                 tap += seg;
                 in_chunk += seg;
                 if (in_chunk == chunk_taps || (slab == nslab - 1 && tap == taps)) {
-                    if (leader) mma_commit(&acc_full[buf]);
+                    mma_commit_warp(&acc_full[buf]);
                     ++gc;
                     in_chunk = 0;
                 }
                 if (!resident) {
-                    if (leader) mma_commit(&b_empty[bs]);
+                    mma_commit_warp(&b_empty[bs]);
                     if (++bs == nbstages) {
                         bs = 0;
                         b_ph ^= 1u;
@@ -560,16 +555,16 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                 }
             }
             if (!ok) break;
-            if (leader) mma_commit(&a_empty[stage]);
+            mma_commit_warp(&a_empty[stage]);
             if (++stage == nstages) {
                 stage = 0;
                 a_ph ^= 1u;
             }
         }
-        if (leader && resident && nt_run_ends(a, t)) mma_commit(&b_empty[0]);
+        if (resident && nt_run_ends(a, t)) mma_commit_warp(&b_empty[0]);
     }
     // every issued MMA completes before TMEM is released
-    if (leader) mma_commit(done);
+    mma_commit_warp(done);
     warp_wait(done, 0, status);
 }
 
@@ -680,10 +675,7 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
             ybase + (static_cast<long long>(g.img) * pix_per_img + (pix_ok ? p : 0)) * out_row_bytes;
         for (int ch = 0; ch < nchunks; ++ch) {
             const int buf = gc % nbuf;
-            int okw = 1;  // warp-uniform bounded wait
-            if (lane == 0) okw = mbar_wait(&acc_full[buf], (full_ph >> buf) & 1u, status) ? 1 : 0;
-            okw = __shfl_sync(0xffffffffu, okw, 0);
-            if (!okw) return;
+            if (!warp_wait(&acc_full[buf], (full_ph >> buf) & 1u, status)) return;
             full_ph ^= 1u << buf;
             tc_fence_after();
             const uint32_t acc_addr = lane_addr + buf * NT;

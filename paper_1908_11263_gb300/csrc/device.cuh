@@ -11,10 +11,9 @@
 namespace qnn {
 
 // A bounded wait gives up after this many SM clock cycles (about two seconds at
-// GB300 clocks); each mbarrier poll may park the thread for at most
-// kSuspendHintNs, and the hardware wakes it as soon as the phase completes.
+// GB300 clocks).  Each mbarrier try_wait may park the thread for a bounded,
+// system-defined time, and the hardware wakes it as soon as the phase completes.
 constexpr long long kWaitLimitCycles = 4000000000ll;
-constexpr uint32_t kSuspendHintNs = 1000000u;
 
 __device__ __forceinline__ void report(int *status, int code) { atomicCAS(status, 0, code); }
 
@@ -46,12 +45,12 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
-__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity)
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
         : "r"(smem_addr(bar)), "r"(parity)
@@ -59,43 +58,25 @@ __device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity)
     return ok != 0;
 }
 
-__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendHintNs)
-        : "memory");
-    return ok != 0;
-}
-
-// Slow path of mbar_wait: polls with the non-blocking test and a short sleep
-// between polls until the phase completes or `limit_cycles` SM cycles pass
-// (then records QNN_ETIMEOUT and returns false).  Out of line so the many wait
-// sites stay small in the instruction cache.
-static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity, int *status, long long limit_cycles)
+// Warp-collective bounded wait: every lane of a converged warp calls it and
+// every lane observes the phase completion itself (so each has the acquire
+// ordering of the barrier).  All lanes poll with try_wait, which parks them in
+// hardware until the phase completes: a hand-off between warps then takes on
+// the order of a hundred cycles, where a single polling lane, a sleep between
+// polls or a shuffle of the result each add more.  Returns false on every lane
+// (and records QNN_ETIMEOUT in *status) once `limit_cycles` SM cycles pass.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *bar, uint32_t parity, int *status,
+                                               long long limit_cycles = kWaitLimitCycles)
 {
     const long long t0 = clock64();
     while (true) {
-        if (mbar_test(bar, parity)) return true;
-        __nanosleep(32);
-        if (clock64() - t0 > limit_cycles) {
-            report(status, QNN_ETIMEOUT);
+        const bool ok = mbar_try_wait(bar, parity);
+        if (__all_sync(0xffffffffu, ok)) return true;
+        if (__any_sync(0xffffffffu, clock64() - t0 > limit_cycles)) {
+            if ((threadIdx.x & 31) == 0) report(status, QNN_ETIMEOUT);
             return false;
         }
     }
-}
-
-// Waits for the phase with the given parity to complete.  Returns false (and
-// records QNN_ETIMEOUT in *status) when `limit_cycles` SM cycles pass first.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *status,
-                                          long long limit_cycles = kWaitLimitCycles)
-{
-    if (mbar_test(bar, parity)) return true;
-    return mbar_wait_slow(bar, parity, status, limit_cycles);
 }
 
 // ------------------------------------------------------------------ bulk copy (TMA, untiled)
@@ -158,6 +139,33 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar)
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                      smem_addr(bar))
                  : "memory");
+}
+
+// Warp-collective forms: every lane of a converged warp executes them and
+// elect.sync (full mask, so always the same lane) issues the operation.  The
+// loop around them then stays converged, its descriptor arithmetic stays
+// warp-uniform, and single-thread issue runs at the shared-memory operand rate
+// instead of paying for a divergent region per MMA.
+__device__ __forceinline__ void mma_f16_ss_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_warp(uint64_t *bar)
+{
+    asm volatile(
+        "{\n\t.reg .pred e;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(
+            smem_addr(bar))
+        : "memory");
 }
 
 // 32 lanes x 32 bits, 16 consecutive columns per thread.
