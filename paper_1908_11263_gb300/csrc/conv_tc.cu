@@ -71,6 +71,29 @@ constexpr uint32_t kCopyChunk = 32768;    // bytes per bulk copy instruction
 constexpr int kMaxAccBufs = 4;
 constexpr int kMaxTaps = 64;  // kh * kw limit of the tensor-core kernel
 
+// Division by a runtime constant d in [1, 2^32) for 32-bit numerators:
+// q = floor(n * m / 2^64) with m = ceil(2^64 / d).  Exact: m * d = 2^64 + e with
+// 0 <= e < d, so n * m / 2^64 = n / d + n * e / (d * 2^64), and the second term
+// is below 1/d for n < 2^32, too small to carry past the next integer.  m = 0
+// stands for d = 1.
+struct FastDiv {
+    unsigned long long m;
+    uint32_t d;
+};
+
+FastDiv make_fastdiv(uint32_t d)
+{
+    FastDiv f;
+    f.d = d;
+    f.m = d <= 1 ? 0ull : (~0ull / d) + 1ull;
+    return f;
+}
+
+__device__ __forceinline__ int fdiv(int n, const FastDiv &f)
+{
+    return f.m == 0ull ? n : static_cast<int>(__umul64hi(static_cast<unsigned long long>(n), f.m));
+}
+
 // Per-channel compression constants (two records per channel, see the prep kernel).
 //   rec0 = {lam2, kappa, shift, mode}   rec1 = {beta, ulo, uhi, lambda}
 enum { kModeWide = 0, kModeClamp = 1, kModeDirect = 2 };
@@ -91,6 +114,7 @@ struct TcArgs {
     uint32_t off_raw, off_stages, off_chan, off_bar;
     uint32_t tmem_cols;
     int *status;
+    FastDiv fd_per_nt, fd_tpi, fd_ow, fd_w;  // n * tiles_per_img, tiles_per_img, ow, w
     uint32_t tap_a16[kMaxTaps];  // per tap (i, j): A offset j*copy + i*ow positions, in 16-byte units
 };
 
@@ -108,14 +132,14 @@ __device__ __forceinline__ TileGeo tile_geo(const TcArgs &a, int t)
 {
     const int per_nt = a.n * a.tiles_per_img;  // total tiles < 2^31 (checked by the planner)
     TileGeo g;
-    g.nt = t / per_nt;
+    g.nt = fdiv(t, a.fd_per_nt);
     const int rem = t - g.nt * per_nt;
-    g.img = rem / a.tiles_per_img;
+    g.img = fdiv(rem, a.fd_tpi);
     g.ti = rem - g.img * a.tiles_per_img;
     const int p0 = g.ti * kTileM;
-    g.oy_a = p0 / a.ow;
+    g.oy_a = fdiv(p0, a.fd_ow);
     g.d0 = p0 - g.oy_a * a.ow;
-    const int out_rows = min((g.d0 + kTileM + a.ow - 1) / a.ow, a.oh - g.oy_a);
+    const int out_rows = min(fdiv(g.d0 + kTileM + a.ow - 1, a.fd_ow), a.oh - g.oy_a);
     g.rows = min(a.rows_max, out_rows + a.kh - 1);
     const int iy0 = g.oy_a - a.ph;
     g.r_lo = min(g.rows, max(0, -iy0));
@@ -123,7 +147,7 @@ __device__ __forceinline__ TileGeo tile_geo(const TcArgs &a, int t)
     return g;
 }
 
-__device__ __forceinline__ int tile_nt(const TcArgs &a, int t) { return t / (a.n * a.tiles_per_img); }
+__device__ __forceinline__ int tile_nt(const TcArgs &a, int t) { return fdiv(t, a.fd_per_nt); }
 
 __device__ __forceinline__ bool nt_run_starts(const TcArgs &a, int t)
 {
@@ -232,96 +256,147 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint4 v)
     asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w));
 }
 
+// Predicated 128-bit shared store (no branch around it).
+__device__ __forceinline__ void sts128_if(bool pred, uint32_t addr, uint4 v)
+{
+    asm volatile(
+        "{\n\t.reg .pred q;\n\t"
+        "setp.ne.b32 q, %5, 0;\n\t"
+        "@q st.shared.v4.b32 [%0], {%1,%2,%3,%4};\n\t}" ::"r"(addr),
+        "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(static_cast<int>(pred)));
+}
+
 // ---------------------------------------------------------------- converters (warps 0-3)
 
-// Rows of the window that lie outside the image read as activation 0.
-template <int BITS>
-__device__ __noinline__ void zero_rows(uint32_t stage, int r_lo, int r_hi, int rows, int ow, int kw, int lg,
-                                       uint32_t copy_bytes, uint32_t chunk_stride)
+// Which column items a converter thread owns, fixed for the whole kernel.  A
+// column item is one (8-channel group gq, pixel x) pair of a staged row, x
+// fastest, so consecutive threads store consecutive 16-byte positions.  When a
+// row has fewer than 128 items the 128 threads split into `nphase` row phases.
+struct ConvMap {
+    int ci0, cstep;  // first column item and stride
+    int rp, nphase;  // first row and row stride
+};
+
+__device__ __forceinline__ ConvMap conv_map(int ncol)
 {
-    const int groups = 1 << lg;
+    const int t = threadIdx.x;  // 0..127
+    ConvMap m;
+    if (ncol <= 128) {
+        m.nphase = 128 / ncol;
+        m.rp = t / ncol;
+        m.ci0 = m.rp < m.nphase ? t - m.rp * ncol : ncol;  // threads past the last phase stay idle
+        m.cstep = ncol;
+        if (m.rp >= m.nphase) m.rp = 0;
+    } else {
+        m.nphase = 1;
+        m.rp = 0;
+        m.ci0 = t;
+        m.cstep = 128;
+    }
+    return m;
+}
+
+// Loads 8 channels of one pixel from a staged raw row and widens them to the
+// staged fp16 encoding (padding value when `ok` is false).
+template <int BITS>
+__device__ __forceinline__ uint4 load_cvt(const uint8_t *p, bool ok, bool vec, const uint8_t *row, int e0, int c0, int c)
+{
     const uint32_t padv = pad_half2<BITS>();
-    const uint4 pad4 = make_uint4(padv, padv, padv, padv);
-    const int zrows = r_lo + (rows - r_hi);
-    const int per_row = ow * groups * kw;
-    for (int it = threadIdx.x; it < zrows * per_row; it += 128) {
-        const int zr = it / per_row;
-        const int rem = it - zr * per_row;
-        const int r = zr < r_lo ? zr : r_hi + (zr - r_lo);
-        const int ox = rem % ow;
-        const int rest = rem / ow;
-        const int gq = rest & (groups - 1);
-        const int j = rest >> lg;
-        sts128(stage + j * copy_bytes + gq * chunk_stride + (r * ow + ox) * 16, pad4);
+    uint4 v = make_uint4(padv, padv, padv, padv);
+    if (ok) {
+        if (!vec) v = cvt_generic<BITS>(row, e0, c0, c);
+        else if (BITS == 8) v = cvt_u8x8(*reinterpret_cast<const uint2 *>(p));
+        else if (BITS == 4) v = cvt_u4x8(*reinterpret_cast<const uint32_t *>(p));
+        else v = cvt_u2x8(*reinterpret_cast<const uint16_t *>(p));
+    }
+    return v;
+}
+
+// Stores one converted pixel into the copies j < NJ whose predicate is set
+// (copy j holds the pixel one position further left per j).
+template <int NJ>
+__device__ __forceinline__ void store_copies(uint8_t *dst, uint32_t jstep, const bool (&pj)[5], const uint4 &v)
+{
+#pragma unroll
+    for (int j = 0; j < NJ; ++j)
+        if (pj[j]) *reinterpret_cast<uint4 *>(dst + j * jstep) = v;
+}
+
+// Rows rp, rp + nph, ... < rows of one column item: four rows per pass (their
+// loads in flight together), then the remaining rows one at a time.
+template <int BITS, int NJ>
+__device__ __forceinline__ void convert_rows(const uint8_t *src, uint8_t *dst, int rp, int nph, int rows, int r_lo,
+                                             int r_hi, bool has_data, bool vec, uint32_t row_bytes, uint32_t row_out,
+                                             uint32_t jstep, const bool (&pj)[5], const uint8_t *raw, int e0, int c0,
+                                             int c)
+{
+    // src / dst point at row rp; src is only dereferenced for rows inside the image
+    const uint32_t src_step = row_bytes * nph, dst_step = row_out * nph;
+    int r = rp;
+    for (; r + 3 * nph < rows; r += 4 * nph) {
+        uint4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int rr = r + u * nph;
+            const bool ok = rr >= r_lo && rr < r_hi && has_data;
+            v[u] = load_cvt<BITS>(src + u * src_step, ok, vec, raw + (rr - r_lo) * row_bytes, e0, c0, c);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) store_copies<NJ>(dst + u * dst_step, jstep, pj, v[u]);
+        src += 4 * src_step;
+        dst += 4 * dst_step;
+    }
+    for (; r < rows; r += nph) {
+        const bool ok = r >= r_lo && r < r_hi && has_data;
+        const uint4 v = load_cvt<BITS>(src, ok, vec, raw + (r - r_lo) * row_bytes, e0, c0, c);
+        store_copies<NJ>(dst, jstep, pj, v);
+        src += src_step;
+        dst += dst_step;
     }
 }
 
-// One (tile, channel slab): raw rows in shared memory -> kw fp16 copies.  Each
-// warp takes whole input rows; within a row, eight consecutive lanes handle
-// eight consecutive pixels of one 8-channel group, so every 128-bit store
-// phase writes 128 contiguous bytes and no division by the width is needed.
+// One (tile, channel slab): staged raw rows -> kw fp16 copies, where copy j
+// holds input pixel (r, ox + j - pw) at position r * ow + ox.  Each thread owns
+// fixed column items (see conv_map) and walks the tile's staged rows for them:
+// per row one load, one conversion and one store per copy that holds the pixel.
+// Rows outside the image store the encoded zero.  Positions of columns that
+// fall outside the image are never written (they keep the encoded zero
+// written at kernel start).
 template <int BITS>
-__device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *raw, uint8_t *smem_out, uint32_t stage,
-                                              const TileGeo &g, int slab, bool vec)
+__device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *raw, uint8_t *stage, const TileGeo &g,
+                                              int slab, bool vec, const ConvMap &mp)
 {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int lg = a.log2_groups;
-    const int groups = 1 << lg;
+    const int ncol = a.w << a.log2_groups;
     const int cb = a.c * BITS / 8;  // packed bytes per pixel
-    const int w = a.w, c = a.c, ow = a.ow, pw = a.pw, kw = a.kw, cs = a.cs;
-    const uint32_t row_bytes = a.row_bytes, chunk_stride = a.chunk_stride, jstep = a.copy_bytes - 16;
-    const int row_items = ((w + 7) >> 3) << (3 + lg);
-    const uint32_t padv = pad_half2<BITS>();
-    const uint4 pad4 = make_uint4(padv, padv, padv, padv);
-    for (int r = g.r_lo + warp; r < g.r_hi; r += 4) {
-        const uint8_t *raw_row = raw + (r - g.r_lo) * row_bytes;
-        const uint32_t out_row = stage + r * ow * 16;  // byte offset within the stage area
-        for (int base = lane; base < row_items; base += 64) {
-            int ix[2], gg[2];
-            uint2 rv[2];
+    const uint32_t jstep = a.copy_bytes - 16;
+    const uint32_t row_out = static_cast<uint32_t>(a.ow) * 16;
+    for (int ci = mp.ci0; ci < ncol; ci += mp.cstep) {
+        const int gq = fdiv(ci, a.fd_w);
+        const int x = ci - gq * a.w;
+        const int c0 = slab * a.cs + gq * 8;
+        // copies j in [jlo, jhi] hold this pixel (their column x + pw - j lies in [0, ow))
+        const int jlo = max(0, x + a.pw - a.ow + 1), jhi = min(a.kw - 1, x + a.pw);
+        bool pj[5];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {  // both loads first
-                const int it = base + u * 32;
-                gg[u] = (it >> 3) & (groups - 1);
-                ix[u] = ((it >> (3 + lg)) << 3) + (it & 7);
-                rv[u] = make_uint2(0, 0);
-                const int c0 = slab * cs + gg[u] * 8;
-                if (it < row_items && ix[u] < w && vec && c0 < c) {
-                    const uint8_t *p = raw_row + ix[u] * cb + c0 * BITS / 8;
-                    if (BITS == 8) rv[u] = *reinterpret_cast<const uint2 *>(p);
-                    else if (BITS == 4) rv[u].x = *reinterpret_cast<const uint32_t *>(p);
-                    else rv[u].x = *reinterpret_cast<const uint16_t *>(p);
-                }
+        for (int j = 0; j < 5; ++j) pj[j] = j >= jlo && j <= jhi;
+        const int rp = mp.rp;
+        const uint8_t *src = raw + (rp - g.r_lo) * static_cast<int>(a.row_bytes) + x * cb + c0 * BITS / 8;
+        uint8_t *dst = stage + gq * a.chunk_stride + (x + a.pw) * 16 + rp * row_out;
+        if (a.kw <= 3)
+            convert_rows<BITS, 3>(src, dst, rp, mp.nphase, g.rows, g.r_lo, g.r_hi, c0 < a.c, vec, a.row_bytes, row_out,
+                                  jstep, pj, raw, x * a.c, c0, a.c);
+        else if (a.kw <= 5)
+            convert_rows<BITS, 5>(src, dst, rp, mp.nphase, g.rows, g.r_lo, g.r_hi, c0 < a.c, vec, a.row_bytes, row_out,
+                                  jstep, pj, raw, x * a.c, c0, a.c);
+        else
+            for (int r = rp; r < g.rows; r += mp.nphase) {  // wide kernels: any kw
+                const bool ok = r >= g.r_lo && r < g.r_hi && c0 < a.c;
+                const uint4 v = load_cvt<BITS>(raw + (r - g.r_lo) * static_cast<int>(a.row_bytes) + x * cb + c0 * BITS / 8,
+                                               ok, vec, raw + (r - g.r_lo) * static_cast<int>(a.row_bytes), x * a.c, c0, a.c);
+                uint8_t *d = stage + gq * a.chunk_stride + (x + a.pw) * 16 + r * row_out;
+                for (int j = jlo; j <= jhi; ++j) *reinterpret_cast<uint4 *>(d + j * jstep) = v;
             }
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const int it = base + u * 32;
-                if (it >= row_items || ix[u] >= w) continue;
-                const int c0 = slab * cs + gg[u] * 8;
-                uint4 v = pad4;
-                if (c0 < c) {
-                    if (!vec) v = cvt_generic<BITS>(raw_row, ix[u] * c, c0, c);
-                    else if (BITS == 8) v = cvt_u8x8(rv[u]);
-                    else if (BITS == 4) v = cvt_u4x8(rv[u].x);
-                    else v = cvt_u2x8(rv[u].x);
-                }
-                // copy j holds this pixel at column ix + pw - j (predicated stores, no branches)
-                uint8_t *dst = smem_out + out_row + gg[u] * chunk_stride + (ix[u] + pw) * 16;
-#pragma unroll
-                for (int j = 0; j < 5; ++j) {
-                    const int ox = ix[u] + pw - j;
-                    if (j < kw && ox >= 0 && ox < ow) *reinterpret_cast<uint4 *>(dst + j * jstep) = v;
-                }
-                for (int j = 5; j < kw; ++j) {
-                    const int ox = ix[u] + pw - j;
-                    if (ox >= 0 && ox < ow) *reinterpret_cast<uint4 *>(dst + j * jstep) = v;
-                }
-            }
-        }
     }
-    if (g.r_lo > 0 || g.rows > g.r_hi)
-        zero_rows<BITS>(smem_addr(smem_out) + stage, g.r_lo, g.r_hi, g.rows, a.ow, a.kw, a.log2_groups, a.copy_bytes,
-                        a.chunk_stride);
 }
 
 template <int BITS>
@@ -330,6 +405,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
 {
     const uint32_t stages_base = smem_addr(smem + a.off_stages);
     const bool vec = (a.c % 8) == 0;
+    const ConvMap mp = conv_map(a.w << a.log2_groups);
     // encoded zero everywhere once: padding columns are never written afterwards
     {
         const uint32_t padv = pad_half2<BITS>();
@@ -345,7 +421,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
         const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         for (int slab = 0; slab < a.nslab; ++slab) {
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
-            convert_stage<BITS>(a, raw, smem + a.off_stages, stage * a.stage_bytes, g, slab, vec);
+            convert_stage<BITS>(a, raw, smem + a.off_stages + stage * a.stage_bytes, g, slab, vec, mp);
             fence_proxy_async_smem();
             mbar_arrive(&a_full[stage]);
             if (++stage == a.stages) {
@@ -945,7 +1021,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
     TcPlan p{};
     p.ok = false;
     if (s.sh != 1 || s.sw != 1 || s.oh <= 0 || s.ow <= 0) return p;
-    if (s.kh * s.kw > kMaxTaps) return p;
+    if (s.kh * s.kw > kMaxTaps || s.kw > 32) return p;  // per-tap table; 32-bit copy mask
     const long long row_bytes = static_cast<long long>(s.w) * s.c * s.bits / 8;
     if (row_bytes % 16 != 0 || row_bytes > (1 << 20)) return p;  // rows move as whole bulk copies
     const int mp16 = (s.m + 15) / 16 * 16;
@@ -1078,6 +1154,10 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.off_raw = plan.off_raw; a.off_stages = plan.off_stages; a.off_chan = plan.off_chan;
     a.off_bar = plan.off_bar;
     a.tmem_cols = plan.tmem_cols;
+    a.fd_per_nt = make_fastdiv(static_cast<uint32_t>(s.n * plan.tiles_per_img));
+    a.fd_tpi = make_fastdiv(static_cast<uint32_t>(plan.tiles_per_img));
+    a.fd_ow = make_fastdiv(static_cast<uint32_t>(s.ow));
+    a.fd_w = make_fastdiv(static_cast<uint32_t>(s.w));
     for (int i = 0; i < s.kh; ++i)
         for (int j = 0; j < s.kw; ++j)
             a.tap_a16[i * s.kw + j] = (j * plan.copy_bytes) / 16 + static_cast<uint32_t>(i * s.ow);
