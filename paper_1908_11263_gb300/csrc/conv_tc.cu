@@ -62,9 +62,13 @@ namespace qnn {
 namespace {
 
 constexpr int kTileM = 128;
-constexpr int kWarps = 11;
+// Warp roles: converters 0-3, epilogue 4-11 (two warps per TMEM lane
+// quarter, one per column half), MMA issuer 12, input-row loader 13, filter
+// loader 14.
+constexpr int kConvWarps = 4, kEpiWarps = 8;
+constexpr int kMmaWarp = 12, kRawWarp = 13, kBWarp = 14;
+constexpr int kWarps = 15;
 constexpr int kThreads = kWarps * 32;
-constexpr int kMmaWarp = 8, kRawWarp = 9, kBWarp = 10;
 constexpr uint32_t kMagic = 0x4B400000u;  // bits of 1.5 * 2^23
 constexpr int kMaxSmem = 232448;          // 227 KB opt-in dynamic shared memory per block
 constexpr uint32_t kCopyChunk = 32768;    // bytes per bulk copy instruction
@@ -93,6 +97,12 @@ __device__ __forceinline__ int fdiv(int n, const FastDiv &f)
 {
     return f.m == 0ull ? n : static_cast<int>(__umul64hi(static_cast<unsigned long long>(n), f.m));
 }
+
+// Per-A-stage record the converter publishes with a_full for the MMA warp:
+// bits 0-15 hold the tile's first pixel column d0, and two flags mark the first
+// and last tile of a run that shares one resident filter set.
+constexpr uint32_t kInfoRunStart = 1u << 30, kInfoRunEnd = 1u << 31;
+constexpr int kMaxStages = 4;
 
 // Per-channel compression constants (two records per channel, see the prep kernel).
 //   rec0 = {lam2, kappa, shift, mode}   rec1 = {beta, ulo, uhi, lambda}
@@ -401,7 +411,7 @@ __device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *ra
 
 template <int BITS>
 __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
-                               uint64_t *a_full, uint64_t *a_empty)
+                               uint64_t *a_full, uint64_t *a_empty, volatile uint32_t *stage_info)
 {
     const uint32_t stages_base = smem_addr(smem + a.off_stages);
     const bool vec = (a.c % 8) == 0;
@@ -417,11 +427,14 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
     uint32_t r_ph = 0, a_ph = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
         const TileGeo g = tile_geo(a, t);
+        const uint32_t info = static_cast<uint32_t>(g.d0) | (nt_run_starts(a, t) ? kInfoRunStart : 0u) |
+                              (nt_run_ends(a, t) ? kInfoRunEnd : 0u);
         if (!warp_wait(&raw_full[rs], r_ph, a.status)) return;
         const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         for (int slab = 0; slab < a.nslab; ++slab) {
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
             convert_stage<BITS>(a, raw, smem + a.off_stages + stage * a.stage_bytes, g, slab, vec, mp);
+            if (threadIdx.x == 0) stage_info[stage] = info;  // released by this thread's arrive below
             fence_proxy_async_smem();
             mbar_arrive(&a_full[stage]);
             if (++stage == a.stages) {
@@ -552,7 +565,8 @@ __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t
 
 __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *a_full,
                                          uint64_t *a_empty, uint64_t *b_full, uint64_t *b_empty, uint64_t *acc_full,
-                                         uint64_t *acc_empty, uint64_t *done, uint32_t idesc, int nt_cols)
+                                         uint64_t *acc_empty, uint64_t *done, const volatile uint32_t *stage_info,
+                                         uint32_t idesc, int nt_cols)
 {
     const uint32_t b_lbo = nt_cols * 16;
     const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
@@ -569,23 +583,30 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
     const int chunk_taps = a.chunk_mmas / ksteps, taps = a.kh * a.kw;
     const int nbuf = a.nbuf, nslab = a.nslab, nstages = a.stages, nbstages = a.b_stages;
     int *const status = a.status;
-    int stage = 0, bs = 0, gc = 0;
+    int stage = 0, bs = 0, buf = 0;
     uint32_t a_ph = 0, b_ph = 0, empty_ph = 0;
     bool ok = true;
+    // The tile sequence matches the converter's; the tile's pixel offset and
+    // filter-run flags come with each stage (no per-tile geometry here).
     for (int t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x) {
-        const TileGeo g = tile_geo(a, t);
-        if (resident && nt_run_starts(a, t)) {
-            if (!warp_wait(&b_full[0], b_ph, status)) break;
-            b_ph ^= 1u;
-        }
-        int in_chunk = 0, buf = 0;
+        int in_chunk = 0;
+        uint32_t info = 0;
         for (int slab = 0; slab < nslab && ok; ++slab) {
             if (!warp_wait(&a_full[stage], a_ph, status)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const uint32_t abase = stages16 + stage * stage16 + g.d0;
+            info = stage_info[stage];
+            if (slab == 0 && resident && (info & kInfoRunStart)) {
+                if (!warp_wait(&b_full[0], b_ph, status)) {
+                    ok = false;
+                    break;
+                }
+                b_ph ^= 1u;
+                tc_fence_after();
+            }
+            const uint32_t abase = stages16 + stage * stage16 + (info & 0xFFFFu);
             int tap = 0;
             while (tap < taps) {
                 uint32_t bbase = b16 + slab * slab_b16;
@@ -599,7 +620,6 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                     seg = 1;
                 }
                 if (in_chunk == 0) {
-                    buf = gc % nbuf;
                     if (!warp_wait(&acc_empty[buf], (empty_ph >> buf) & 1u, status)) {
                         ok = false;
                         break;
@@ -619,7 +639,7 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                 in_chunk += seg;
                 if (in_chunk == chunk_taps || (slab == nslab - 1 && tap == taps)) {
                     mma_commit_warp(&acc_full[buf]);
-                    ++gc;
+                    if (++buf == nbuf) buf = 0;
                     in_chunk = 0;
                 }
                 if (!resident) {
@@ -637,7 +657,7 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                 a_ph ^= 1u;
             }
         }
-        if (resident && nt_run_ends(a, t)) mma_commit_warp(&b_empty[0]);
+        if (ok && resident && (info & kInfoRunEnd)) mma_commit_warp(&b_empty[0]);
     }
     // every issued MMA completes before TMEM is released
     mma_commit_warp(done);
@@ -667,60 +687,148 @@ __device__ __noinline__ uint32_t compress_slow(uint32_t s, int4 r0, int4 r1, uin
     return compress64(u, r0.y, r1.w, r0.z, top);
 }
 
-// Compression (Sec. III-A) of 16 raw sums of one pixel, Q-bit packing
-// (Sec. IV-A) and store of the channels below m.  Direct channels (the common
-// case) compute clip(((s * kappa + lam2) mod 2^32) >> shift): the prep kernel
+// Saturating pack of two results (cvt.pack.sat): returns
+// (upper << 2Q) | (clip(hi) << Q) | clip(lo) with clip to [0, 2^Q - 1], the
+// clip of the compression step (Sec. III-A) fused with the Q-bit packing of
+// Sec. IV-A.
+template <int BITS>
+__device__ __forceinline__ uint32_t pack2_sat(int hi, int lo, uint32_t upper)
+{
+    uint32_t d;
+    if (BITS == 8) asm("cvt.pack.sat.u8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(hi), "r"(lo), "r"(upper));
+    else if (BITS == 4) asm("cvt.pack.sat.u4.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(hi), "r"(lo), "r"(upper));
+    else asm("cvt.pack.sat.u2.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(hi), "r"(lo), "r"(upper));
+    return d;
+}
+
+// Compression (Sec. III-A) of G raw sums of one pixel, Q-bit packing (Sec.
+// IV-A) and store of the channels below m.  Direct channels (the common case)
+// compute ((s * kappa + lam2) mod 2^32) >> shift and clip it: the prep kernel
 // has proved that (acc + bias) * kappa + lambda stays inside int32 for every
 // accumulator the layer can produce, and folded bias, the staging offset and
 // the accumulator pre-load into lam2, so the wrapped 32-bit value is exact.
-template <int BITS>
-__device__ __forceinline__ void compress_store16(const uint32_t (&s)[16], const int4 *rec0, const int4 *rec1,
-                                                 bool direct, int m_first, int valid, uint8_t *dst)
+template <int BITS, int G>
+__device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *rec0, const int4 *rec1, bool direct,
+                                               int m_first, int valid, uint8_t *dst)
 {
-    constexpr uint32_t top = (1u << BITS) - 1u;
-    constexpr int kWords = 16 * BITS / 32;
-    uint32_t packed[kWords];
-#pragma unroll
-    for (int wd = 0; wd < kWords; ++wd) packed[wd] = 0;
+    int y[G];
     if (direct) {
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
+        for (int k = 0; k < G; ++k) {
             const int4 r0 = rec0[m_first + k];
-            const int32_t t = static_cast<int32_t>(s[k] * static_cast<uint32_t>(r0.y) + static_cast<uint32_t>(r0.x))
-                              >> r0.z;
-            const uint32_t yv = static_cast<uint32_t>(min(max(t, 0), static_cast<int32_t>(top)));
-            packed[(k * BITS) / 32] |= yv << ((k * BITS) % 32);
+            y[k] = static_cast<int32_t>(s[k] * static_cast<uint32_t>(r0.y) + static_cast<uint32_t>(r0.x)) >> r0.z;
         }
     } else {
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-            const uint32_t yv = compress_slow(s[k], rec0[m_first + k], rec1[m_first + k], top);
-            packed[(k * BITS) / 32] |= yv << ((k * BITS) % 32);
-        }
+        for (int k = 0; k < G; ++k)
+            y[k] = static_cast<int>(compress_slow(s[k], rec0[m_first + k], rec1[m_first + k], (1u << BITS) - 1u));
     }
-    constexpr int kBytes = 16 * BITS / 8;
-    if (valid >= 16 && (reinterpret_cast<uintptr_t>(dst) % kBytes) == 0) {
-        if (BITS == 8) *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
-        else if (BITS == 4) *reinterpret_cast<uint2 *>(dst) = make_uint2(packed[0], packed[1]);
-        else *reinterpret_cast<uint32_t *>(dst) = packed[0];
+    constexpr int kPer = 32 / BITS;                   // results per 32-bit word
+    constexpr int kWords = (G * BITS + 31) / 32;
+    uint32_t packed[kWords];
+#pragma unroll
+    for (int wd = 0; wd < kWords; ++wd) {
+        uint32_t t = 0;
+#pragma unroll
+        for (int k = kPer - 2; k >= 0; k -= 2) {  // highest pair first; it ends in the top bits
+            const int e = wd * kPer + k;
+            if (e < G) t = pack2_sat<BITS>(y[e + 1], y[e], t);
+        }
+        packed[wd] = t;
+    }
+    constexpr int kBytes = G * BITS / 8;
+    if (valid >= G && (reinterpret_cast<uintptr_t>(dst) % kBytes) == 0) {
+        if (kBytes == 16) *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        else if (kBytes == 8) *reinterpret_cast<uint2 *>(dst) = make_uint2(packed[0], packed[kWords > 1 ? 1 : 0]);
+        else if (kBytes == 4) *reinterpret_cast<uint32_t *>(dst) = packed[0];
+        else *reinterpret_cast<uint16_t *>(dst) = static_cast<uint16_t>(packed[0]);
     } else {
-        const int nbytes = min(valid, 16) * BITS / 8;
+        const int nbytes = min(valid, G) * BITS / 8;
 #pragma unroll
         for (int b = 0; b < kBytes; ++b)
             if (b < nbytes) dst[b] = static_cast<uint8_t>(packed[b / 4] >> (8 * (b % 4)));
     }
 }
 
+// TMEM access in steps of 16 (or, for 8-column warps, 8) columns.
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t *v)
+{
+    if (N == 8) {
+        uint32_t t[8];
+        tmem_ld8(taddr, t);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[k] = t[k];
+    } else {
+#pragma unroll
+        for (int c = 0; c < N; c += 16) {
+            uint32_t t[16];
+            tmem_ld16(taddr + c, t);
+#pragma unroll
+            for (int k = 0; k < 16; ++k) v[c + k] = t[k];
+        }
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t *v)
+{
+    if (N == 8) {
+        uint32_t t[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t[k] = v[k];
+        tmem_st8(taddr, t);
+    } else {
+#pragma unroll
+        for (int c = 0; c < N; c += 16) {
+            uint32_t t[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) t[k] = v[c + k];
+            tmem_st16(taddr + c, t);
+        }
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_fill_cols(uint32_t taddr, uint32_t value)
+{
+    if (N == 8) {
+        tmem_st8_fill(taddr, value);
+    } else {
+#pragma unroll
+        for (int c = 0; c < N; c += 16) tmem_st16_fill(taddr + c, value);
+    }
+}
+
+// Releases an accumulator buffer: this warp's TMEM stores are complete before
+// one lane arrives (the barrier counts one arrival per epilogue warp).
+__device__ __forceinline__ void release_acc(uint64_t *bar)
+{
+    tmem_wait_st();
+    tc_fence_before();
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
+// Epilogue warps: warp w reads TMEM lane quarter w % 4 (tile rows = output
+// pixels) and one half of the NT columns.  Per chunk it loads its columns in
+// batches of up to 32 with one wait each, adds the running integer sums, puts
+// the accumulator pre-load back and releases the buffer before the
+// compression arithmetic, so the MMA warp can refill it meanwhile.
 template <int BITS, int NT>
 __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
-                              uint64_t *acc_empty)
+                                              uint64_t *acc_empty)
 {
-    // TMEM columns: nbuf fp32 accumulators of NT columns each, then (when K
-    // needs several chunks) NT columns of running integer sums.
-    const int quarter = (threadIdx.x >> 5) & 3;
+    constexpr int CW = NT / 2;                  // columns of this warp
+    constexpr int BATCH = CW < 32 ? CW : 32;   // columns per TMEM wait
+    constexpr int G = CW < 16 ? CW : 16;       // channels per compression group
+    const int warp = threadIdx.x >> 5;
+    const int quarter = warp & 3;
+    const int half = (warp - kConvWarps) >> 2;
     const int lane = threadIdx.x & 31;
     const int row = quarter * 32 + lane;  // tile row = output pixel within the tile
-    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16);
+    const int col0 = half * CW;
+    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + col0;
     const uint32_t sum_addr = lane_addr + a.nbuf * NT;
     const int mp = a.n_ntiles * NT;
     const int4 *rec0 = reinterpret_cast<const int4 *>(smem + a.off_chan);
@@ -732,54 +840,56 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
     uint8_t *const ybase = a.y;
     int *const status = a.status;
 
-    for (int col = 0; col < nbuf * NT; col += 16) tmem_st16_fill(lane_addr + col, kMagic);
+    for (int b = 0; b < nbuf; ++b) tmem_fill_cols<CW>(lane_addr + b * NT, kMagic);
     tmem_wait_st();
     tc_fence_before();
-    for (int b = 0; b < nbuf; ++b) mbar_arrive(&acc_empty[b]);
+    __syncwarp();
+    if (lane == 0)
+        for (int b = 0; b < nbuf; ++b) mbar_arrive(&acc_empty[b]);
 
     uint32_t full_ph = 0;
-    int gc = 0;
+    int buf = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
         const TileGeo g = tile_geo(a, t);
         // Pixels past the end of the image are computed but not stored.  TMEM
         // accesses are warp-collective, so every lane executes them; only the
         // store depends on the lane's pixel.
         const int p = g.ti * kTileM + row;
-        const int m0 = g.nt * NT;
+        const int m0 = g.nt * NT + col0;
         const bool pix_ok = p < pix_per_img;
         uint8_t *dst_row =
             ybase + (static_cast<long long>(g.img) * pix_per_img + (pix_ok ? p : 0)) * out_row_bytes;
         for (int ch = 0; ch < nchunks; ++ch) {
-            const int buf = gc % nbuf;
             if (!warp_wait(&acc_full[buf], (full_ph >> buf) & 1u, status)) return;
             full_ph ^= 1u << buf;
             tc_fence_after();
             const uint32_t acc_addr = lane_addr + buf * NT;
             const bool last = ch == nchunks - 1;
-#pragma unroll 1
-            for (int col = 0; col < NT; col += 16) {
-                uint32_t v[16], prev[16];
-                tmem_ld16(acc_addr + col, v);
-                if (ch > 0) tmem_ld16(sum_addr + col, prev);
+            uint32_t v[CW];
+#pragma unroll
+            for (int b0 = 0; b0 < CW; b0 += BATCH) {
+                uint32_t prev[BATCH];
+                tmem_ld_cols<BATCH>(acc_addr + b0, v + b0);
+                if (ch > 0) tmem_ld_cols<BATCH>(sum_addr + b0, prev);
                 tmem_wait_ld();
                 if (ch > 0) {
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) v[k] += prev[k];
+                    for (int k = 0; k < BATCH; ++k) v[b0 + k] += prev[k];
                 }
-                tmem_st16_fill(acc_addr + col, kMagic);
-                if (!last) {
-                    tmem_st16(sum_addr + col, v);
-                } else {
-                    const int valid = m - (m0 + col);  // same for the whole warp
-                    if (pix_ok && valid > 0)
-                        compress_store16<BITS>(v, rec0, rec1, gdirect[(m0 + col) >> 4] != 0, m0 + col, valid,
-                                               dst_row + (m0 + col) * BITS / 8);
+                tmem_fill_cols<BATCH>(acc_addr + b0, kMagic);
+                if (!last) tmem_st_cols<BATCH>(sum_addr + b0, v + b0);
+            }
+            release_acc(&acc_empty[buf]);
+            if (++buf == nbuf) buf = 0;
+            if (last && pix_ok) {
+#pragma unroll
+                for (int c = 0; c < CW; c += G) {
+                    const int valid = m - (m0 + c);  // same for the whole warp
+                    if (valid > 0)
+                        compress_store<BITS, G>(v + c, rec0, rec1, gdirect[(m0 + c) >> 4] != 0, m0 + c, valid,
+                                                dst_row + (m0 + c) * BITS / 8);
                 }
             }
-            tmem_wait_st();
-            tc_fence_before();
-            mbar_arrive(&acc_empty[buf]);
-            ++gc;
         }
     }
 }
@@ -799,6 +909,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     uint64_t *acc_empty = acc_full + kMaxAccBufs;
     uint64_t *done = acc_empty + kMaxAccBufs;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    volatile uint32_t *stage_info = tmem_slot + 1;  // kMaxStages words
     const int warp = threadIdx.x >> 5;
 
     if (warp == kMmaWarp) {
@@ -817,7 +928,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
             }
             for (int b = 0; b < kMaxAccBufs; ++b) {
                 mbar_init(&acc_full[b], 1);
-                mbar_init(&acc_empty[b], 128);
+                mbar_init(&acc_empty[b], kEpiWarps);
             }
             mbar_init(done, 1);
             fence_mbar_init();
@@ -825,13 +936,14 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
         __syncwarp();
         tmem_alloc(tmem_slot, a.tmem_cols);
         tmem_relinquish();
-    } else if (warp >= 4 && warp < 8) {
+    } else if (warp >= kConvWarps && warp < kConvWarps + kEpiWarps) {
         // compression records, plus one "all direct" flag per 16-channel group
         int4 *chan = reinterpret_cast<int4 *>(smem + a.off_chan);
         const int mp = a.n_ntiles * NT;
-        for (int i = threadIdx.x - 128; i < 2 * mp; i += 128) chan[i] = a.chan[i];
+        const int et = threadIdx.x - kConvWarps * 32, ne = kEpiWarps * 32;
+        for (int i = et; i < 2 * mp; i += ne) chan[i] = a.chan[i];
         uint8_t *gdirect = reinterpret_cast<uint8_t *>(chan + 2 * mp);
-        for (int gi = threadIdx.x - 128; gi < mp / 16; gi += 128) {
+        for (int gi = et; gi < mp / 16; gi += ne) {
             int all = 1;
             for (int k = 0; k < 16; ++k) all &= a.chan[gi * 16 + k].w == kModeDirect;
             gdirect[gi] = static_cast<uint8_t>(all);
@@ -842,12 +954,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    if (warp < 4) {
-        converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
-    } else if (warp < 8) {
+    if (warp < kConvWarps) {
+        converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty, stage_info);
+    } else if (warp < kConvWarps + kEpiWarps) {
         epilogue_role<BITS, NT>(a, smem, tmem_base, acc_full, acc_empty);
     } else if (warp == kMmaWarp) {
-        mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+        mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info,
                  idesc_f16_f32(kTileM, NT), NT);
     } else if (warp == kRawWarp) {
         raw_loader_role(a, smem, raw_full, raw_empty);
@@ -1064,7 +1176,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     const uint32_t off_chan = off_stages + stages * stage_bytes;
                     const uint32_t off_bar = off_chan + chan_bytes;
                     const uint32_t nbars = 2 * p.raw_stages + 2 * stages + 2 * b_stages + 2 * kMaxAccBufs + 1;
-                    const uint32_t total = off_bar + nbars * 8 + 16;
+                    const uint32_t total = off_bar + nbars * 8 + 4 + 4 * kMaxStages;  // TMEM slot, stage records
                     if (total > static_cast<uint32_t>(kMaxSmem)) continue;
                     p.cs = cs;
                     p.nslab = p.c_pad / cs;
