@@ -72,7 +72,7 @@ constexpr int kThreads = kWarps * 32;
 constexpr uint32_t kMagic = 0x4B400000u;  // bits of 1.5 * 2^23
 constexpr int kMaxSmem = 232448;          // 227 KB opt-in dynamic shared memory per block
 constexpr uint32_t kCopyChunk = 32768;    // bytes per bulk copy instruction
-constexpr int kMaxAccBufs = 4;
+constexpr int kMaxAccGroups = 4;
 constexpr int kMaxTaps = 64;  // kh * kw limit of the tensor-core kernel
 
 // Division by a runtime constant d in [1, 2^32) for 32-bit numerators:
@@ -119,7 +119,7 @@ struct TcArgs {
     int total_tiles;
     int rows_max, p_alloc;
     int stages, raw_stages, b_stages, b_resident;
-    int mmas_per_tile, chunk_mmas, nchunks, nbuf;
+    int mmas_per_tile, chunk_mmas, nchunks, grp_chunks, ngroups, nsg;
     uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, chunk_stride;
     uint32_t off_raw, off_stages, off_chan, off_bar;
     uint32_t tmem_cols;
@@ -581,15 +581,16 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
     // resident filters: tap t of slab s sits at t * c_pad/8 chunks; streamed: each tap has its own tile
     const uint32_t tap_b16 = resident ? (a.c_pad / 8) * nt_cols : 0;
     const int chunk_taps = a.chunk_mmas / ksteps, taps = a.kh * a.kw;
-    const int nbuf = a.nbuf, nslab = a.nslab, nstages = a.stages, nbstages = a.b_stages;
+    const int nslab = a.nslab, nstages = a.stages, nbstages = a.b_stages;
+    const int grp_chunks = a.grp_chunks, ngroups = a.ngroups, nchunks = a.nchunks;
     int *const status = a.status;
-    int stage = 0, bs = 0, buf = 0;
+    int stage = 0, bs = 0, grp = 0;
     uint32_t a_ph = 0, b_ph = 0, empty_ph = 0;
     bool ok = true;
     // The tile sequence matches the converter's; the tile's pixel offset and
     // filter-run flags come with each stage (no per-tile geometry here).
     for (int t = blockIdx.x; t < a.total_tiles && ok; t += gridDim.x) {
-        int in_chunk = 0;
+        int in_chunk = 0, chunk = 0, sub = 0;  // MMAs into the current chunk, chunk of the tile, buffer in the group
         uint32_t info = 0;
         for (int slab = 0; slab < nslab && ok; ++slab) {
             if (!warp_wait(&a_full[stage], a_ph, status)) {
@@ -619,16 +620,16 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                     bbase = b16 + bs * btile16 - tap * tap_b16;
                     seg = 1;
                 }
-                if (in_chunk == 0) {
-                    if (!warp_wait(&acc_empty[buf], (empty_ph >> buf) & 1u, status)) {
+                if (in_chunk == 0 && sub == 0) {  // a new accumulator group
+                    if (!warp_wait(&acc_empty[grp], (empty_ph >> grp) & 1u, status)) {
                         ok = false;
                         break;
                     }
-                    empty_ph ^= 1u << buf;
+                    empty_ph ^= 1u << grp;
                     tc_fence_after();
                 }
                 seg = min(seg, chunk_taps - in_chunk);
-                const uint32_t d = tmem_base + buf * nt_cols;
+                const uint32_t d = tmem_base + (grp * grp_chunks + sub) * nt_cols;
                 if (ksteps == 1)
                     issue_taps<1>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
                 else if (ksteps == 2)
@@ -637,10 +638,14 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                     issue_taps<4>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
                 tap += seg;
                 in_chunk += seg;
-                if (in_chunk == chunk_taps || (slab == nslab - 1 && tap == taps)) {
-                    mma_commit_warp(&acc_full[buf]);
-                    if (++buf == nbuf) buf = 0;
+                if (in_chunk == chunk_taps || (slab == nslab - 1 && tap == taps)) {  // chunk complete
                     in_chunk = 0;
+                    ++chunk;
+                    if (++sub == grp_chunks || chunk == nchunks) {  // group complete
+                        mma_commit_warp(&acc_full[grp]);
+                        sub = 0;
+                        if (++grp == ngroups) grp = 0;
+                    }
                 }
                 if (!resident) {
                     mma_commit_warp(&b_empty[bs]);
@@ -752,7 +757,7 @@ __device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *re
 
 // TMEM access in steps of 16 (or, for 8-column warps, 8) columns.
 template <int N>
-__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t *v)
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&v)[N])
 {
     if (N == 8) {
         uint32_t t[8];
@@ -771,7 +776,7 @@ __device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t *v)
 }
 
 template <int N>
-__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t *v)
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&v)[N])
 {
     if (N == 8) {
         uint32_t t[8];
@@ -811,44 +816,48 @@ __device__ __forceinline__ void release_acc(uint64_t *bar)
 }
 
 // Epilogue warps: warp w reads TMEM lane quarter w % 4 (tile rows = output
-// pixels) and one half of the NT columns.  Per chunk it loads its columns in
-// batches of up to 32 with one wait each, adds the running integer sums, puts
-// the accumulator pre-load back and releases the buffer before the
-// compression arithmetic, so the MMA warp can refill it meanwhile.
+// pixels) and one half of the NT columns.  Per accumulator group it adds the
+// group's buffers (the raw fp32 bit patterns, an exact integer sum, see the
+// prep kernel) in batches of up to 32 columns, puts the accumulator pre-load
+// back and releases the group before the compression arithmetic, so the MMA
+// warp can refill it meanwhile.  Tiles that take several groups carry their
+// running sums in TMEM.
 template <int BITS, int NT>
 __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
                                               uint64_t *acc_empty)
 {
     constexpr int CW = NT / 2;                  // columns of this warp
-    constexpr int BATCH = CW < 32 ? CW : 32;   // columns per TMEM wait
+    constexpr int BATCH = CW < 16 ? CW : 16;   // columns per TMEM wait
     constexpr int G = CW < 16 ? CW : 16;       // channels per compression group
+    constexpr int kMaxSrc = 512 / NT / 2 + 1;  // buffers of one group (planner bound) plus the running sums
     const int warp = threadIdx.x >> 5;
     const int quarter = warp & 3;
     const int half = (warp - kConvWarps) >> 2;
     const int lane = threadIdx.x & 31;
     const int row = quarter * 32 + lane;  // tile row = output pixel within the tile
     const int col0 = half * CW;
+    const int grp_chunks = a.grp_chunks, ngroups = a.ngroups, nsg = a.nsg, nchunks = a.nchunks;
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + col0;
-    const uint32_t sum_addr = lane_addr + a.nbuf * NT;
+    const uint32_t sum_addr = lane_addr + ngroups * grp_chunks * NT;
     const int mp = a.n_ntiles * NT;
     const int4 *rec0 = reinterpret_cast<const int4 *>(smem + a.off_chan);
     const int4 *rec1 = rec0 + mp;
     const uint8_t *gdirect = reinterpret_cast<const uint8_t *>(rec1 + mp);  // per 16-channel group
     const int pix_per_img = a.oh * a.ow;
     const int out_row_bytes = a.m * BITS / 8;
-    const int nbuf = a.nbuf, nchunks = a.nchunks, m = a.m;
+    const int m = a.m;
     uint8_t *const ybase = a.y;
     int *const status = a.status;
 
-    for (int b = 0; b < nbuf; ++b) tmem_fill_cols<CW>(lane_addr + b * NT, kMagic);
+    for (int b = 0; b < ngroups * grp_chunks; ++b) tmem_fill_cols<CW>(lane_addr + b * NT, kMagic);
     tmem_wait_st();
     tc_fence_before();
     __syncwarp();
     if (lane == 0)
-        for (int b = 0; b < nbuf; ++b) mbar_arrive(&acc_empty[b]);
+        for (int b = 0; b < ngroups; ++b) mbar_arrive(&acc_empty[b]);
 
     uint32_t full_ph = 0;
-    int buf = 0;
+    int grp = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
         const TileGeo g = tile_geo(a, t);
         // Pixels past the end of the image are computed but not stored.  TMEM
@@ -859,28 +868,44 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
         const bool pix_ok = p < pix_per_img;
         uint8_t *dst_row =
             ybase + (static_cast<long long>(g.img) * pix_per_img + (pix_ok ? p : 0)) * out_row_bytes;
-        for (int ch = 0; ch < nchunks; ++ch) {
-            if (!warp_wait(&acc_full[buf], (full_ph >> buf) & 1u, status)) return;
-            full_ph ^= 1u << buf;
+        for (int sg = 0; sg < nsg; ++sg) {
+            if (!warp_wait(&acc_full[grp], (full_ph >> grp) & 1u, status)) return;
+            full_ph ^= 1u << grp;
             tc_fence_after();
-            const uint32_t acc_addr = lane_addr + buf * NT;
-            const bool last = ch == nchunks - 1;
+            const int nsub = min(grp_chunks, nchunks - sg * grp_chunks);
+            const uint32_t grp_addr = lane_addr + grp * grp_chunks * NT;
+            const bool last = sg == nsg - 1;
             uint32_t v[CW];
 #pragma unroll
-            for (int b0 = 0; b0 < CW; b0 += BATCH) {
-                uint32_t prev[BATCH];
-                tmem_ld_cols<BATCH>(acc_addr + b0, v + b0);
-                if (ch > 0) tmem_ld_cols<BATCH>(sum_addr + b0, prev);
-                tmem_wait_ld();
-                if (ch > 0) {
+            for (int k = 0; k < CW; ++k) v[k] = 0;
+            const int nsrc = nsub + (sg > 0 ? 1 : 0);
 #pragma unroll
-                    for (int k = 0; k < BATCH; ++k) v[b0 + k] += prev[k];
+            for (int sub = 0; sub < kMaxSrc; ++sub) {  // unrolled: v[] stays in registers
+                // the group's buffers, then (for a tile's later groups) its running sums
+                if (sub >= nsrc) break;
+                const bool is_sum = sub == nsub;
+                const uint32_t src = is_sum ? sum_addr : grp_addr + sub * NT;
+#pragma unroll
+                for (int b0 = 0; b0 < CW; b0 += BATCH) {
+                    uint32_t tmp[BATCH];
+                    tmem_ld_cols<BATCH>(src + b0, tmp);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int k = 0; k < BATCH; ++k) v[b0 + k] += tmp[k];
+                    if (!is_sum) tmem_fill_cols<BATCH>(src + b0, kMagic);
                 }
-                tmem_fill_cols<BATCH>(acc_addr + b0, kMagic);
-                if (!last) tmem_st_cols<BATCH>(sum_addr + b0, v + b0);
             }
-            release_acc(&acc_empty[buf]);
-            if (++buf == nbuf) buf = 0;
+            if (!last) {
+#pragma unroll
+                for (int b0 = 0; b0 < CW; b0 += BATCH) {
+                    uint32_t tmp[BATCH];
+#pragma unroll
+                    for (int k = 0; k < BATCH; ++k) tmp[k] = v[b0 + k];
+                    tmem_st_cols<BATCH>(sum_addr + b0, tmp);
+                }
+            }
+            release_acc(&acc_empty[grp]);
+            if (++grp == ngroups) grp = 0;
             if (last && pix_ok) {
 #pragma unroll
                 for (int c = 0; c < CW; c += G) {
@@ -906,8 +931,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     uint64_t *b_full = a_empty + a.stages;
     uint64_t *b_empty = b_full + a.b_stages;
     uint64_t *acc_full = b_empty + a.b_stages;
-    uint64_t *acc_empty = acc_full + kMaxAccBufs;
-    uint64_t *done = acc_empty + kMaxAccBufs;
+    uint64_t *acc_empty = acc_full + kMaxAccGroups;
+    uint64_t *done = acc_empty + kMaxAccGroups;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
     volatile uint32_t *stage_info = tmem_slot + 1;  // kMaxStages words
     const int warp = threadIdx.x >> 5;
@@ -926,7 +951,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
                 mbar_init(&b_full[s], 1);
                 mbar_init(&b_empty[s], 1);
             }
-            for (int b = 0; b < kMaxAccBufs; ++b) {
+            for (int b = 0; b < kMaxAccGroups; ++b) {
                 mbar_init(&acc_full[b], 1);
                 mbar_init(&acc_empty[b], kEpiWarps);
             }
@@ -1175,7 +1200,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     const uint32_t off_stages = off_raw + p.raw_stages * p.raw_bytes;
                     const uint32_t off_chan = off_stages + stages * stage_bytes;
                     const uint32_t off_bar = off_chan + chan_bytes;
-                    const uint32_t nbars = 2 * p.raw_stages + 2 * stages + 2 * b_stages + 2 * kMaxAccBufs + 1;
+                    const uint32_t nbars = 2 * p.raw_stages + 2 * stages + 2 * b_stages + 2 * kMaxAccGroups + 1;
                     const uint32_t total = off_bar + nbars * 8 + 4 + 4 * kMaxStages;  // TMEM slot, stage records
                     if (total > static_cast<uint32_t>(kMaxSmem)) continue;
                     p.cs = cs;
@@ -1208,11 +1233,22 @@ TcPlan plan_conv_tc(const ConvShape &s)
         p.nchunks = (units + per - 1) / per;
         p.chunk_mmas = per * ksteps;
     }
-    // accumulator ring: up to four buffers, plus the integer sums when K takes several chunks
-    const int sum_cols = p.nchunks > 1 ? p.nt : 0;
-    p.nbuf = std::min(kMaxAccBufs, (512 - sum_cols) / p.nt);
+    // Accumulator groups: a tile's chunks go to grp_chunks TMEM buffers that
+    // complete together (one hand-off per group).  When two groups of all the
+    // tile's chunks do not fit in the 512 columns, a tile takes several groups
+    // and carries its running integer sums in NT more columns.
+    int sum_cols = 0;
+    if (2 * p.nchunks * p.nt <= 512) {
+        p.grp_chunks = p.nchunks;
+        p.nsg = 1;
+    } else {
+        p.grp_chunks = std::max(1, (512 - p.nt) / (2 * p.nt));
+        p.nsg = (p.nchunks + p.grp_chunks - 1) / p.grp_chunks;
+        sum_cols = p.nt;
+    }
+    p.ngroups = std::min(kMaxAccGroups, (512 - sum_cols) / (p.grp_chunks * p.nt));
     p.tmem_cols = 32;
-    while (p.tmem_cols < static_cast<uint32_t>(p.nbuf * p.nt + sum_cols)) p.tmem_cols *= 2;
+    while (p.tmem_cols < static_cast<uint32_t>(p.ngroups * p.grp_chunks * p.nt + sum_cols)) p.tmem_cols *= 2;
     p.tiles_per_img = static_cast<int>((static_cast<long long>(s.oh) * s.ow + kTileM - 1) / kTileM);
     p.total_tiles = static_cast<long long>(p.n_ntiles) * s.n * p.tiles_per_img;
     if (p.total_tiles >= (1ll << 31)) return p;
@@ -1258,7 +1294,7 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.stages = plan.stages; a.raw_stages = plan.raw_stages; a.b_stages = plan.b_stages;
     a.b_resident = plan.b_resident;
     a.mmas_per_tile = plan.mmas_per_tile; a.chunk_mmas = plan.chunk_mmas; a.nchunks = plan.nchunks;
-    a.nbuf = plan.nbuf;
+    a.grp_chunks = plan.grp_chunks; a.ngroups = plan.ngroups; a.nsg = plan.nsg;
     a.row_bytes = plan.row_bytes; a.raw_bytes = plan.raw_bytes;
     a.b_bytes = plan.b_bytes; a.b_tile_bytes = plan.b_tile_bytes;
     a.copy_bytes = plan.copy_bytes; a.stage_bytes = plan.stage_bytes;

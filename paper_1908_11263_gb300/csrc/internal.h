@@ -46,7 +46,9 @@ struct TcPlan {
     int limit_mmas;     // most MMAs one exact fp32 accumulator chunk may take
     int chunk_mmas;     // MMAs per exact fp32 accumulator chunk (whole taps)
     int nchunks;        // chunks per tile
-    int nbuf;           // TMEM accumulator buffers in the ring
+    int grp_chunks;     // chunks per accumulator group (one TMEM buffer each, completed together)
+    int ngroups;        // accumulator groups in the TMEM ring
+    int nsg;            // groups per tile (more than one: running sums kept in TMEM)
     uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, smem_bytes, tmem_cols;
     uint32_t off_raw, off_stages, off_chan, off_bar;
     size_t workspace_bytes;
