@@ -38,7 +38,28 @@ from paper_1908_11263_gb300 import inputs  # noqa: E402
 
 L2_BYTES = 129 * 1024 * 1024
 WORKLOAD = "conv3x3_16x16x32_to_64_int8_n512"
+INT8_IMMA_TOPS = 151.6
 METRIC = "qconv_hwc GMAC/s (16x16x32 -> 64, 3x3, stride 1, pad 1, INT-8, batch 512)"
+
+
+PROFILE = os.path.join(ROOT, "profiles", "conv_tc_kernel_conv3x3_16x16x32to64_int8_n512.md")
+KERNEL_SOURCES = ("conv_tc.cu", "device.cuh", "internal.h")
+
+
+def measured_traffic():
+    """DRAM bytes per launch of the timed convolution kernel, from the committed
+    ncu summary, or None when the kernel's sources changed since that capture."""
+    import hashlib
+    try:
+        line = next(l for l in open(PROFILE) if l.startswith("traffic:"))
+        rec = json.loads(line[len("traffic:"):])
+    except (OSError, StopIteration, ValueError):
+        return None
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_1908_11263_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return rec["dram_bytes_per_launch"] if h.hexdigest() == rec["source_sha256"] else None
 
 
 def peaks():
@@ -79,6 +100,12 @@ def max_over_ranks(value: float, world: int, device=None) -> float:
     t = torch.tensor([value], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_rate(units_per_rank_step: float, world: int, steps: int, t_max: float) -> float:
+    """Units every rank processed, per second of the slowest rank's time (weak
+    scaling: each rank runs `steps` steps of the same size on its own shard)."""
+    return world * units_per_rank_step * steps / t_max
 
 
 # ---------------------------------------------------------------------------- clocks
@@ -250,7 +277,7 @@ def run_ours(args, world, rank, local):
     alg_bytes = layer.algorithmic_bytes()
     result = None
     if rank == 0:
-        gmacs = world * macs / (t_max / k) / 1e9
+        gmacs = whole_job_rate(macs, world, k, t_max) / 1e9
         result = {
             "metric": METRIC,
             "value": round(gmacs, 1),
@@ -282,9 +309,13 @@ def run_ours(args, world, rank, local):
                 "algorithmic_flops": flops,
                 "algorithmic_bytes": alg_bytes,
                 "hbm_frac_at_this_time": round(alg_bytes / kernel_s / 1e9 / pk["hbm_gbs"], 4),
-                "traffic": None,
+                "traffic": measured_traffic(),
             },
-            "e2e": {"value": round(world * macs / (t_e2e / e2e_k) / 1e9, 1), "unit": "GMAC/s",
+            # the only INT8 tensor path on sm_103a is the warp-level mma.sync IMMA (no tcgen05 kind::i8);
+            # its rate on this GPU, measured with m16n8k32 u8*s8 MMAs from all SMs, is context only
+            "int8_tensor_ref": {"peak_tops": INT8_IMMA_TOPS, "frac": round(achieved_tflops / INT8_IMMA_TOPS, 3),
+                                "source": "measured mma.sync.m16n8k32 u8*s8 rate, all SMs, GB300"},
+            "e2e": {"value": round(whole_job_rate(macs, world, e2e_k, t_e2e) / 1e9, 1), "unit": "GMAC/s",
                     "h2d_bytes_per_step": int(xh.numel()), "d2h_bytes_per_step": int(yh.numel()),
                     "steps": e2e_k},
             "clocks": clocks,

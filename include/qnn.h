@@ -218,6 +218,19 @@ qnn_status unpack_subbyte(const void *src, int8_t *dst, int64_t count, int32_t b
  */
 qnn_status qnn_device_status(void *stream);
 
+/*
+ * Diagnostics: runs the library's bounded-wait failure path on the GPU.  One
+ * warp waits on an mbarrier that nothing arrives on; after `limit_cycles` SM
+ * cycles the wait gives up, records QNN_ETIMEOUT in the device status word and
+ * the kernel returns, leaving the context usable.  Every wait inside the
+ * library's kernels is bounded the same way (a wait that never completes
+ * turns into QNN_ETIMEOUT, not a hang).  The paper has no counterpart; this
+ * exists so that the failure path can be tested without faulting a GPU.
+ * limit_cycles must lie in [1, 2^31); QNN_EINVAL otherwise.  Read the result
+ * with qnn_device_status(stream).
+ */
+qnn_status qnn_selftest_wait_timeout(int64_t limit_cycles, void *stream);
+
 /* Static description of a status code. */
 const char *qnn_status_string(qnn_status s);
 

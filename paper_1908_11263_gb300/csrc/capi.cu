@@ -131,6 +131,18 @@ void *noalloc_scratch_ptr()
     return cache[dev];
 }
 
+// One warp waits on a barrier that nothing arrives on (bounded by `limit`).
+__global__ void selftest_timeout_kernel(int *status, long long limit)
+{
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    mbar_wait_warp(&bar, 0, status, limit);
+}
+
 }  // namespace
 }  // namespace qnn
 
@@ -288,6 +300,15 @@ qnn_status unpack_subbyte(const void *src, int8_t *dst, int64_t count, int32_t b
     if (count % (8 / bits)) return QNN_EUNSUPPORTED;
     return from_cuda(launch_unpack(static_cast<const uint8_t *>(src), dst, count, bits, is_signed ? 1 : 0,
                                    static_cast<cudaStream_t>(stream)));
+}
+
+qnn_status qnn_selftest_wait_timeout(int64_t limit_cycles, void *stream)
+{
+    if (limit_cycles < 1 || limit_cycles >= (1ll << 31)) return QNN_EINVAL;
+    int *status = device_status_ptr();
+    if (!status) return QNN_ECUDA;
+    selftest_timeout_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(status, limit_cycles);
+    return from_cuda(cudaGetLastError());
 }
 
 qnn_status qnn_device_status(void *stream)

@@ -25,7 +25,8 @@ NOALLOC_SCRATCH_BYTES = 2 << 20  # QNN_NOALLOC_SCRATCH_BYTES
 ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
-            "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc")
+            "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
+            "qnn_selftest_wait_timeout")
 
 
 class QnnError(RuntimeError):
@@ -81,6 +82,8 @@ def load(build_if_missing: bool = False):
         lib.pack_subbyte.restype = I32
         lib.unpack_subbyte.argtypes = [P, P, I64, I32, I32, P]
         lib.unpack_subbyte.restype = I32
+        lib.qnn_selftest_wait_timeout.argtypes = [I64, P]
+        lib.qnn_selftest_wait_timeout.restype = I32
         lib.qnn_device_status.argtypes = [P]
         lib.qnn_device_status.restype = I32
         lib.qnn_status_string.argtypes = [I32]
@@ -314,6 +317,11 @@ def unpack_subbyte(src, bits, signed, *, out=None, stream=None):
     st = load().unpack_subbyte(_ptr(src), _ptr(out), out.numel(), bits, int(bool(signed)), _stream(stream))
     _check(st, "unpack_subbyte")
     return out
+
+
+def selftest_wait_timeout(limit_cycles: int, stream=None):
+    """Enqueue the bounded-wait failure self-test (see qnn_selftest_wait_timeout)."""
+    _check(load().qnn_selftest_wait_timeout(int(limit_cycles), _stream(stream)), "qnn_selftest_wait_timeout")
 
 
 def device_status(stream=None):
