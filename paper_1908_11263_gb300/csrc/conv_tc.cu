@@ -563,6 +563,76 @@ __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t
     }
 }
 
+// MMA issue for the common case: filters resident and one channel slab per
+// tile.  Each accumulator group's chunks are contiguous tap ranges issued
+// back to back, with no per-segment bookkeeping between them.  The tensor
+// pipe queues only a few MMAs, so any work this warp does between MMAs shows
+// up as idle tensor cycles; this loop keeps that work to the waits and commits.
+template <int KSTEPS>
+__device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem, uint32_t tmem_base,
+                                                  uint64_t *a_full, uint64_t *a_empty, uint64_t *b_full,
+                                                  uint64_t *b_empty, uint64_t *acc_full, uint64_t *acc_empty,
+                                                  uint64_t *done, const volatile uint32_t *stage_info, uint32_t idesc,
+                                                  int nt_cols)
+{
+    const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
+    const uint64_t b_tmpl = smem_desc(0, nt_cols * 16, 128);
+    const uint32_t stages16 = smem_addr(smem + a.off_stages) >> 4;
+    const uint32_t b16 = smem_addr(smem) >> 4;
+    const uint32_t stage16 = a.stage_bytes >> 4;
+    const uint32_t a_step = 2 * (a.chunk_stride >> 4), b_step = 2 * nt_cols;
+    const uint32_t tap_b16 = (a.c_pad / 8) * nt_cols;
+    const int chunk_taps = a.chunk_mmas / KSTEPS, taps = a.kh * a.kw;
+    const int ngroups = a.ngroups, grp_chunks = a.grp_chunks, nsg = a.nsg, nchunks = a.nchunks;
+    const int nstages = a.stages;
+    const uint32_t grp_cols = grp_chunks * nt_cols;
+    int *const status = a.status;
+    int stage = 0, grp = 0;
+    uint32_t a_ph = 0, b_ph = 0, empty_ph = 0;
+    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+        if (!warp_wait(&a_full[stage], a_ph, status)) break;
+        tc_fence_after();
+        const uint32_t info = stage_info[stage];
+        if (info & kInfoRunStart) {
+            if (!warp_wait(&b_full[0], b_ph, status)) break;
+            b_ph ^= 1u;
+            tc_fence_after();
+        }
+        const uint32_t abase = stages16 + stage * stage16 + (info & 0xFFFFu);
+        bool ok = true;
+        int t0 = 0;
+        for (int sg = 0; sg < nsg; ++sg) {
+            if (!warp_wait(&acc_empty[grp], (empty_ph >> grp) & 1u, status)) {
+                ok = false;
+                break;
+            }
+            empty_ph ^= 1u << grp;
+            tc_fence_after();
+            uint32_t d = tmem_base + grp * grp_cols;
+            const int last_chunk = min(nchunks, (sg + 1) * grp_chunks);
+            for (int c = sg * grp_chunks; c < last_chunk; ++c) {
+                const int t1 = min(t0 + chunk_taps, taps);
+                issue_taps<KSTEPS>(a, d, a_tmpl, b_tmpl, abase, b16, tap_b16, a_step, b_step, t0, t1, idesc);
+                t0 = t1;
+                d += nt_cols;
+            }
+            mma_commit_warp(&acc_full[grp]);
+            if (++grp == ngroups) grp = 0;
+        }
+        if (!ok) break;
+        mma_commit_warp(&a_empty[stage]);
+        if (++stage == nstages) {
+            stage = 0;
+            a_ph ^= 1u;
+        }
+        if (info & kInfoRunEnd) mma_commit_warp(&b_empty[0]);
+    }
+    // every issued MMA completes before TMEM is released
+    mma_commit_warp(done);
+    warp_wait(done, 0, status);
+}
+
+// MMA issue, general case (streamed filters, or several channel slabs per tile).
 __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *a_full,
                                          uint64_t *a_empty, uint64_t *b_full, uint64_t *b_empty, uint64_t *acc_full,
                                          uint64_t *acc_empty, uint64_t *done, const volatile uint32_t *stage_info,
@@ -984,8 +1054,19 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     } else if (warp < kConvWarps + kEpiWarps) {
         epilogue_role<BITS, NT>(a, smem, tmem_base, acc_full, acc_empty);
     } else if (warp == kMmaWarp) {
-        mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info,
-                 idesc_f16_f32(kTileM, NT), NT);
+        const uint32_t idesc = idesc_f16_f32(kTileM, NT);
+        if (a.b_resident && a.nslab == 1 && a.cs == 32)
+            mma_role_resident<2>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                 stage_info, idesc, NT);
+        else if (a.b_resident && a.nslab == 1 && a.cs == 64)
+            mma_role_resident<4>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                 stage_info, idesc, NT);
+        else if (a.b_resident && a.nslab == 1)
+            mma_role_resident<1>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                 stage_info, idesc, NT);
+        else
+            mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info, idesc,
+                     NT);
     } else if (warp == kRawWarp) {
         raw_loader_role(a, smem, raw_full, raw_empty);
     } else if (warp == kBWarp) {
