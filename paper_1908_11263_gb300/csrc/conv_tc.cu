@@ -64,10 +64,11 @@ namespace {
 constexpr int kTileM = 128;
 // Warp roles: converters 0-3, epilogue 4-11 (two warps per TMEM lane
 // quarter, one per column half), MMA issuer 12, input-row loader 13, filter
-// loader 14.
+// loader 14, second MMA issuer 15 (takes alternate tiles when the whole
+// kernel uses one resident filter set).
 constexpr int kConvWarps = 4, kEpiWarps = 8;
-constexpr int kMmaWarp = 12, kRawWarp = 13, kBWarp = 14;
-constexpr int kWarps = 15;
+constexpr int kMmaWarp = 12, kRawWarp = 13, kBWarp = 14, kMmaWarp2 = 15;
+constexpr int kWarps = 16;
 constexpr int kThreads = kWarps * 32;
 constexpr uint32_t kMagic = 0x4B400000u;  // bits of 1.5 * 2^23
 constexpr int kMaxSmem = 232448;          // 227 KB opt-in dynamic shared memory per block
@@ -125,6 +126,7 @@ struct TcArgs {
     uint32_t tmem_cols;
     int *status;
     FastDiv fd_per_nt, fd_tpi, fd_ow, fd_w;  // n * tiles_per_img, tiles_per_img, ow, w
+    int mma_warps;                            // 2: warps 12 and 15 issue alternate tiles
     uint32_t tap_a16[kMaxTaps];  // per tap (i, j): A offset j*copy + i*ow positions, in 16-byte units
 };
 
@@ -542,7 +544,7 @@ __device__ __forceinline__ void b_loader_role(const TcArgs &a, uint8_t *smem, ui
     else drain_ring(b_full, bs, ph, a.b_stages, issued, a.status);
 }
 
-// ---------------------------------------------------------------- MMA issuer (warp 8)
+// ---------------------------------------------------------------- MMA issuers (warps 12 and 15)
 
 // Issues the MMAs of taps [t0, t1) of one slab: KSTEPS k-steps (16 channels each)
 // per tap.  Called by the whole converged MMA warp (one elected lane issues).
@@ -568,12 +570,17 @@ __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t
 // back to back, with no per-segment bookkeeping between them.  The tensor
 // pipe queues only a few MMAs, so any work this warp does between MMAs shows
 // up as idle tensor cycles; this loop keeps that work to the waits and commits.
+//
+// With two issuers (one filter set for the whole kernel), issuer `sel` takes
+// the CTA's tiles sel, sel + 2, ...; stage, group and their phases follow from
+// the tile's position in the CTA's sequence, so one issuer's waits and commits
+// overlap the other's MMAs.
 template <int KSTEPS>
 __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem, uint32_t tmem_base,
                                                   uint64_t *a_full, uint64_t *a_empty, uint64_t *b_full,
                                                   uint64_t *b_empty, uint64_t *acc_full, uint64_t *acc_empty,
                                                   uint64_t *done, const volatile uint32_t *stage_info, uint32_t idesc,
-                                                  int nt_cols)
+                                                  int nt_cols, int sel, int nsel)
 {
     const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
     const uint64_t b_tmpl = smem_desc(0, nt_cols * 16, 128);
@@ -587,13 +594,19 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
     const int nstages = a.stages;
     const uint32_t grp_cols = grp_chunks * nt_cols;
     int *const status = a.status;
-    int stage = 0, grp = 0;
-    uint32_t a_ph = 0, b_ph = 0, empty_ph = 0;
-    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
-        if (!warp_wait(&a_full[stage], a_ph, status)) break;
+    // the two issuers' `done` commits both count (the barrier expects nsel arrivals)
+    uint32_t b_ph = 0;
+    if (nsel > 1) {  // one filter set for the whole kernel: both issuers wait for it once
+        if (!warp_wait(&b_full[0], 0, status)) nsel = 0;
+        tc_fence_after();
+    }
+    for (int i = sel, t = blockIdx.x + sel * gridDim.x; nsel > 0 && t < a.total_tiles;
+         i += nsel, t += nsel * gridDim.x) {
+        const int stage = i % nstages;
+        if (!warp_wait(&a_full[stage], (i / nstages) & 1, status)) break;
         tc_fence_after();
         const uint32_t info = stage_info[stage];
-        if (info & kInfoRunStart) {
+        if (nsel == 1 && (info & kInfoRunStart)) {
             if (!warp_wait(&b_full[0], b_ph, status)) break;
             b_ph ^= 1u;
             tc_fence_after();
@@ -602,11 +615,12 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
         bool ok = true;
         int t0 = 0;
         for (int sg = 0; sg < nsg; ++sg) {
-            if (!warp_wait(&acc_empty[grp], (empty_ph >> grp) & 1u, status)) {
+            const int gc = i * nsg + sg;  // groups used so far by this CTA
+            const int grp = gc % ngroups;
+            if (!warp_wait(&acc_empty[grp], (gc / ngroups) & 1, status)) {
                 ok = false;
                 break;
             }
-            empty_ph ^= 1u << grp;
             tc_fence_after();
             uint32_t d = tmem_base + grp * grp_cols;
             const int last_chunk = min(nchunks, (sg + 1) * grp_chunks);
@@ -617,15 +631,10 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
                 d += nt_cols;
             }
             mma_commit_warp(&acc_full[grp]);
-            if (++grp == ngroups) grp = 0;
         }
         if (!ok) break;
         mma_commit_warp(&a_empty[stage]);
-        if (++stage == nstages) {
-            stage = 0;
-            a_ph ^= 1u;
-        }
-        if (info & kInfoRunEnd) mma_commit_warp(&b_empty[0]);
+        if (nsel == 1 && (info & kInfoRunEnd)) mma_commit_warp(&b_empty[0]);
     }
     // every issued MMA completes before TMEM is released
     mma_commit_warp(done);
@@ -739,7 +748,7 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
     warp_wait(done, 0, status);
 }
 
-// ---------------------------------------------------------------- epilogue (warps 4-7)
+// ---------------------------------------------------------------- epilogue (warps 4-11)
 
 // Compression of one integer sum u = acc + bias in 64-bit arithmetic.
 __device__ __noinline__ uint32_t compress64(int32_t u, int32_t kappa, int32_t lambda, int32_t shift, uint32_t top)
@@ -1025,7 +1034,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
                 mbar_init(&acc_full[b], 1);
                 mbar_init(&acc_empty[b], kEpiWarps);
             }
-            mbar_init(done, 1);
+            mbar_init(done, a.mma_warps);
             fence_mbar_init();
         }
         __syncwarp();
@@ -1053,17 +1062,18 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
         converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty, stage_info);
     } else if (warp < kConvWarps + kEpiWarps) {
         epilogue_role<BITS, NT>(a, smem, tmem_base, acc_full, acc_empty);
-    } else if (warp == kMmaWarp) {
+    } else if (warp == kMmaWarp || (warp == kMmaWarp2 && a.mma_warps == 2)) {
         const uint32_t idesc = idesc_f16_f32(kTileM, NT);
+        const int sel = warp == kMmaWarp ? 0 : 1;
         if (a.b_resident && a.nslab == 1 && a.cs == 32)
             mma_role_resident<2>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                 stage_info, idesc, NT);
+                                 stage_info, idesc, NT, sel, a.mma_warps);
         else if (a.b_resident && a.nslab == 1 && a.cs == 64)
             mma_role_resident<4>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                 stage_info, idesc, NT);
+                                 stage_info, idesc, NT, sel, a.mma_warps);
         else if (a.b_resident && a.nslab == 1)
             mma_role_resident<1>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                 stage_info, idesc, NT);
+                                 stage_info, idesc, NT, sel, a.mma_warps);
         else
             mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info, idesc,
                      NT);
@@ -1387,6 +1397,8 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.fd_tpi = make_fastdiv(static_cast<uint32_t>(plan.tiles_per_img));
     a.fd_ow = make_fastdiv(static_cast<uint32_t>(s.ow));
     a.fd_w = make_fastdiv(static_cast<uint32_t>(s.w));
+    // two MMA issuers when every tile of the kernel uses the same resident filter set
+    a.mma_warps = (plan.b_resident && plan.nslab == 1 && plan.n_ntiles == 1) ? 2 : 1;
     for (int i = 0; i < s.kh; ++i)
         for (int j = 0; j < s.kw; ++j)
             a.tap_a16[i * s.kw + j] = (j * plan.copy_bytes) / 16 + static_cast<uint32_t>(i * s.ow);
