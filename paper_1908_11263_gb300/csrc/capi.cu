@@ -204,7 +204,7 @@ qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const v
     st = check_workspace(plan, workspace, workspace_bytes);
     if (st != QNN_OK) return st;
     return from_cuda(launch_conv_tc_run(plan, s, static_cast<const uint8_t *>(x), static_cast<uint8_t *>(y),
-                                        workspace, static_cast<cudaStream_t>(stream)));
+                                        workspace, static_cast<cudaStream_t>(stream), false));
 }
 
 qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias, const int16_t *kappa,
@@ -227,7 +227,7 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
         ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
                      d->shift, static_cast<uint8_t *>(y)};
         cudaError_t e = launch_conv_tc_prep(plan, s, p, workspace, cs);
-        if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, workspace, cs);
+        if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, workspace, cs, true);
         return from_cuda(e);
     }
     if (s.n == 0) return QNN_OK;
@@ -258,7 +258,7 @@ qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *
     ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
                  d->shift, static_cast<uint8_t *>(y)};
     cudaError_t e = launch_conv_tc_prep(plan, s, p, scratch, cs);
-    if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, scratch, cs);
+    if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, scratch, cs, true);
     return from_cuda(e);
 }
 

@@ -508,6 +508,7 @@ __device__ __forceinline__ void raw_loader_role(const TcArgs &a, uint8_t *smem, 
 // tile (resident), or one [nt x cs] tile per (slab, tap) step (streamed).
 __device__ __forceinline__ void b_loader_role(const TcArgs &a, uint8_t *smem, uint64_t *b_full, uint64_t *b_empty, int nt_cols)
 {
+    pdl_wait();  // the filters come from the preparation kernel, which may still be running
     int bs = 0;
     uint32_t ph = 0;
     int issued = 0;
@@ -884,6 +885,12 @@ __device__ __forceinline__ void tmem_fill_cols(uint32_t taddr, uint32_t value)
     }
 }
 
+// Barrier among the epilogue warps only (named barrier 1).
+__device__ __forceinline__ void epi_barrier()
+{
+    asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+}
+
 // Releases an accumulator buffer: this warp's TMEM stores are complete before
 // one lane arrives (the barrier counts one arrival per epilogue warp).
 __device__ __forceinline__ void release_acc(uint64_t *bar)
@@ -934,6 +941,21 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
     __syncwarp();
     if (lane == 0)
         for (int b = 0; b < ngroups; ++b) mbar_arrive(&acc_empty[b]);
+    // compression records (written by the preparation kernel, which may still be
+    // running), plus one "all direct" flag per 16-channel group
+    pdl_wait();
+    {
+        int4 *chan = reinterpret_cast<int4 *>(smem + a.off_chan);
+        const int et = threadIdx.x - kConvWarps * 32, ne = kEpiWarps * 32;
+        for (int i = et; i < 2 * mp; i += ne) chan[i] = a.chan[i];
+        uint8_t *gd = reinterpret_cast<uint8_t *>(chan + 2 * mp);
+        for (int gi = et; gi < mp / 16; gi += ne) {
+            int all = 1;
+            for (int k = 0; k < 16; ++k) all &= a.chan[gi * 16 + k].w == kModeDirect;
+            gd[gi] = static_cast<uint8_t>(all);
+        }
+        epi_barrier();
+    }
 
     uint32_t full_ph = 0;
     int grp = 0;
@@ -1040,18 +1062,6 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
         __syncwarp();
         tmem_alloc(tmem_slot, a.tmem_cols);
         tmem_relinquish();
-    } else if (warp >= kConvWarps && warp < kConvWarps + kEpiWarps) {
-        // compression records, plus one "all direct" flag per 16-channel group
-        int4 *chan = reinterpret_cast<int4 *>(smem + a.off_chan);
-        const int mp = a.n_ntiles * NT;
-        const int et = threadIdx.x - kConvWarps * 32, ne = kEpiWarps * 32;
-        for (int i = et; i < 2 * mp; i += ne) chan[i] = a.chan[i];
-        uint8_t *gdirect = reinterpret_cast<uint8_t *>(chan + 2 * mp);
-        for (int gi = et; gi < mp / 16; gi += ne) {
-            int all = 1;
-            for (int k = 0; k < 16; ++k) all &= a.chan[gi * 16 + k].w == kModeDirect;
-            gdirect[gi] = static_cast<uint8_t>(all);
-        }
     }
     tc_fence_before();
     __syncthreads();
@@ -1128,7 +1138,7 @@ __device__ bool saturation_bounds(long long kappa, long long lambda, int s, long
     return in_i32(*ulo * kappa + lambda) && in_i32(*uhi * kappa + lambda);
 }
 
-// One block per (padded) output channel: fp16 filters in the [ntile][k/8][nt][8]
+// One warp per (padded) output channel: fp16 filters in the [ntile][k/8][nt][8]
 // layout of the B operand, and the channel's compression records:
 //   rec0 = {lam2, kappa, shift, mode}, rec1 = {beta, ulo, uhi, lambda}
 // where the epilogue's raw sum s (sum of the chunks' bit patterns) relates to the
@@ -1136,72 +1146,76 @@ __device__ bool saturation_bounds(long long kappa, long long lambda, int s, long
 // (mod 2^32).  Mode "direct" holds when (acc + bias)*kappa + lambda fits int32 for
 // every accumulator this channel's weights can produce (activations in
 // [0, 2^Q-1]); mode "clamp" when the saturation bounds allow a 32-bit form.
+// The kernel lets the convolution that follows it start at once (that kernel
+// waits for these results only where it reads them).
 template <int BITS>
-__global__ void __launch_bounds__(128) conv_tc_prep_kernel(const uint8_t *w, const int32_t *bias, const int16_t *kappa,
+__global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, const int32_t *bias, const int16_t *kappa,
                                                            const int32_t *lambda, const uint8_t *shifts, int shift,
-                                                           int m, int kh, int kw, int c, int c_pad, int k_pad, int nt,
-                                                           int nchunks, uint16_t *wpack, int4 *chan)
+                                                           int m, int mp, int kh, int kw, int c, int c_pad, int k_pad,
+                                                           int nt, int nchunks, uint16_t *wpack, int4 *chan)
 {
-    const int o = blockIdx.x;
-    const int tile = o / nt, col = o % nt;
+    pdl_trigger();
+    const int lane = threadIdx.x & 31;
+    const int o = blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (o >= mp) return;
+    const int tile = o / nt, col = o - tile * nt;
+    const int taps = kh * kw;
     const int slot_of[8] = {0, 2, 4, 6, 1, 3, 5, 7};  // inverse of {0,4,1,5,2,6,3,7}
-    long long sum = 0, pos = 0, neg = 0;
-    for (int k = threadIdx.x; k < k_pad; k += blockDim.x) {
-        const int tap = k / c_pad, cc = k - tap * c_pad;
-        int v = 0;
-        if (o < m && cc < c) {
-            const long long e = (static_cast<long long>(o) * kh * kw + tap) * c + cc;
-            if (BITS == 8) {
-                v = static_cast<int8_t>(w[e]);
-            } else {
-                const int per = 8 / BITS;
-                const int f = (w[e / per] >> ((e % per) * BITS)) & ((1 << BITS) - 1);
-                v = f >= (1 << (BITS - 1)) ? f - (1 << BITS) : f;
+    int sum = 0, pos = 0, neg = 0;  // |sum| <= K * 2^(Q-1) < 2^31 (accumulator bound of the ABI)
+    for (int tap = 0; tap < taps; ++tap) {
+        for (int cc = lane; cc < c_pad; cc += 32) {  // consecutive lanes: consecutive channels and slots
+            int v = 0;
+            if (o < m && cc < c) {
+                const long long e = (static_cast<long long>(o) * taps + tap) * c + cc;
+                if (BITS == 8) {
+                    v = static_cast<int8_t>(w[e]);
+                } else {
+                    constexpr int per = 8 / BITS;
+                    const int f = (w[e / per] >> ((e % per) * BITS)) & ((1 << BITS) - 1);
+                    v = f >= (1 << (BITS - 1)) ? f - (1 << BITS) : f;
+                }
             }
+            sum += v;
+            pos += max(v, 0);
+            neg += min(v, 0);
+            const int k = tap * c_pad + cc;
+            const int slot = BITS == 8 ? (cc & 7) : slot_of[cc & 7];
+            const size_t dst = ((static_cast<size_t>(tile) * (k_pad / 8) + k / 8) * nt + col) * 8 + slot;
+            wpack[dst] = __half_as_ushort(__int2half_rn(v));
         }
-        sum += v;
-        if (v > 0) pos += v;
-        else neg += v;
-        const int slot = BITS == 8 ? (cc & 7) : slot_of[cc & 7];
-        const size_t dst = ((static_cast<size_t>(tile) * (k_pad / 8) + k / 8) * nt + col) * 8 + slot;
-        wpack[dst] = __half_as_ushort(__int2half_rn(v));
     }
-    __shared__ long long red[3][128];
-    red[0][threadIdx.x] = sum;
-    red[1][threadIdx.x] = pos;
-    red[2][threadIdx.x] = neg;
-    __syncthreads();
-    for (int s = 64; s > 0; s >>= 1) {
-        if (threadIdx.x < s)
-            for (int r = 0; r < 3; ++r) red[r][threadIdx.x] += red[r][threadIdx.x + s];
-        __syncthreads();
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) {
+        sum += __shfl_xor_sync(0xffffffffu, sum, d);
+        pos += __shfl_xor_sync(0xffffffffu, pos, d);
+        neg += __shfl_xor_sync(0xffffffffu, neg, d);
     }
-    if (threadIdx.x == 0) {
+    if (lane == 0) {
         int4 r0 = make_int4(0, 0, 0, kModeDirect), r1 = make_int4(0, 0, 0, 0);
         if (o < m) {
             const long long off = (BITS == 8) ? -128 : 1024;  // staged activation = x + off
             const int32_t b = bias ? bias[o] : 0;
-            const uint32_t beta = static_cast<uint32_t>(b) - static_cast<uint32_t>(off * red[0][0]) -
+            const uint32_t beta = static_cast<uint32_t>(b) - static_cast<uint32_t>(off * sum) -
                                   static_cast<uint32_t>(nchunks) * kMagic;
             const int32_t kap = kappa[o], lam = lambda[o], sh = shifts ? shifts[o] : shift;
             const long long top = (1 << BITS) - 1;
             // every accumulator of this channel lies in [top * neg, top * pos]
-            const long long u0 = top * red[2][0] + b, u1 = top * red[1][0] + b;
+            const long long u0 = top * neg + b, u1 = top * pos + b;
             const bool direct = in_i32(u0 * kap + lam) && in_i32(u1 * kap + lam);
-            long long ulo, uhi;
-            const bool clamp = saturation_bounds(kap, lam, sh, top, &ulo, &uhi);
+            long long ulo = 0, uhi = 0;
+            const bool clamp = !direct && saturation_bounds(kap, lam, sh, top, &ulo, &uhi);
             const int mode = direct ? kModeDirect : clamp ? kModeClamp : kModeWide;
             const uint32_t lam2 = beta * static_cast<uint32_t>(kap) + static_cast<uint32_t>(lam);
             r0 = make_int4(static_cast<int32_t>(lam2), kap, sh, mode);
             r1 = make_int4(static_cast<int32_t>(beta), static_cast<int32_t>(ulo), static_cast<int32_t>(uhi), lam);
         }
         chan[o] = r0;
-        chan[gridDim.x + o] = r1;
+        chan[mp + o] = r1;
     }
 }
 
 template <int BITS, int NT>
-cudaError_t launch_tc(const TcArgs &args, int grid, uint32_t smem, cudaStream_t st)
+cudaError_t launch_tc(const TcArgs &args, int grid, uint32_t smem, cudaStream_t st, bool after_prep)
 {
     // the opt-in shared-memory limit is raised once per device, outside any stream capture
     static std::mutex mu;
@@ -1219,18 +1233,33 @@ cudaError_t launch_tc(const TcArgs &args, int grid, uint32_t smem, cudaStream_t 
             raised[dev] = true;
         }
     }
-    kern<<<grid, kThreads, smem, st>>>(args);
-    return cudaGetLastError();
+    if (!after_prep) {
+        kern<<<grid, kThreads, smem, st>>>(args);
+        return cudaGetLastError();
+    }
+    // Right after the preparation kernel: start while it still runs.  Only the
+    // filter loader and the epilogue's record load wait for its results.
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args);
 }
 
 template <int BITS>
-cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, cudaStream_t st)
+cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, cudaStream_t st, bool after_prep)
 {
     switch (nt) {
-        case 16: return launch_tc<BITS, 16>(args, grid, smem, st);
-        case 32: return launch_tc<BITS, 32>(args, grid, smem, st);
-        case 64: return launch_tc<BITS, 64>(args, grid, smem, st);
-        case 128: return launch_tc<BITS, 128>(args, grid, smem, st);
+        case 16: return launch_tc<BITS, 16>(args, grid, smem, st, after_prep);
+        case 32: return launch_tc<BITS, 32>(args, grid, smem, st, after_prep);
+        case 64: return launch_tc<BITS, 64>(args, grid, smem, st, after_prep);
+        case 128: return launch_tc<BITS, 128>(args, grid, smem, st, after_prep);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -1354,9 +1383,10 @@ cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const Co
     uint16_t *wpack = static_cast<uint16_t *>(workspace);
     int4 *chan = reinterpret_cast<int4 *>(static_cast<uint8_t *>(workspace) + chan_offset(plan));
     const int mp = plan.n_ntiles * plan.nt;
-#define QNN_PREP(B)                                                                                               \
-    conv_tc_prep_kernel<B><<<mp, 128, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, s.kh, s.kw, \
-                                               s.c, plan.c_pad, plan.k_pad, plan.nt, plan.nchunks, wpack, chan)
+#define QNN_PREP(B)                                                                                              \
+    conv_tc_prep_kernel<B><<<(mp + 7) / 8, 256, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, \
+                                                         mp, s.kh, s.kw, s.c, plan.c_pad, plan.k_pad, plan.nt,   \
+                                                         plan.nchunks, wpack, chan)
     switch (s.bits) {
         case 8: QNN_PREP(8); break;
         case 4: QNN_PREP(4); break;
@@ -1367,7 +1397,7 @@ cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const Co
 }
 
 cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uint8_t *x, uint8_t *y,
-                               const void *workspace, cudaStream_t st)
+                               const void *workspace, cudaStream_t st, bool after_prep)
 {
     if (s.n == 0) return cudaSuccess;
     TcArgs a{};
@@ -1407,9 +1437,9 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     const long long sms = device_sm_count();
     const int grid = static_cast<int>(std::min<long long>(plan.total_tiles, sms));
     switch (s.bits) {
-        case 8: return launch_tc_bits<8>(plan.nt, a, grid, plan.smem_bytes, st);
-        case 4: return launch_tc_bits<4>(plan.nt, a, grid, plan.smem_bytes, st);
-        default: return launch_tc_bits<2>(plan.nt, a, grid, plan.smem_bytes, st);
+        case 8: return launch_tc_bits<8>(plan.nt, a, grid, plan.smem_bytes, st, after_prep);
+        case 4: return launch_tc_bits<4>(plan.nt, a, grid, plan.smem_bytes, st, after_prep);
+        default: return launch_tc_bits<2>(plan.nt, a, grid, plan.smem_bytes, st, after_prep);
     }
 }
 

@@ -17,6 +17,12 @@ constexpr long long kWaitLimitCycles = 4000000000ll;
 
 __device__ __forceinline__ void report(int *status, int code) { atomicCAS(status, 0, code); }
 
+// Programmatic dependent launch: a primary grid lets the next kernel of the
+// stream start early (pdl_trigger); that kernel calls pdl_wait before it
+// touches the primary's results.  Both are no-ops without such a launch.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t smem_addr(const void *p)
 {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -57,8 +57,10 @@ struct TcPlan {
 TcPlan plan_conv_tc(const ConvShape &s);
 cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
                                 cudaStream_t st);
+// after_prep: launched right after launch_conv_tc_prep on the same stream, so the
+// convolution may start while the preparation kernel still runs.
 cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uint8_t *x, uint8_t *y,
-                               const void *workspace, cudaStream_t st);
+                               const void *workspace, cudaStream_t st, bool after_prep);
 
 // ---- max-pool, fully connected, packing
 cudaError_t launch_maxpool(int n, int h, int w, int c, int k, int s, int bits, const uint8_t *x, uint8_t *y,
