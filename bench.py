@@ -426,6 +426,179 @@ def run_reference(args, world, rank):
     }
 
 
+# ---------------------------------------------------------------------------- per-config sweep
+
+def run_sweep(args):
+    """One JSON line per layer of workloads 1, 3, 4 and 5 (workload 2 is the default run):
+    GMAC/s of qconv_hwc calls and of the convolution kernel alone, each timed from CUDA
+    graphs over rotating buffer sets larger than L2, with the roof that binds the layer
+    (its arithmetic intensity against the measured ridge) and the fraction reached."""
+    import torch
+    from paper_1908_11263_gb300 import qnn
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    qnn.load(build_if_missing=True)
+    pk = peaks()
+    ridge = pk["bf16_tflops"] * 1e12 / (pk["hbm_gbs"] * 1e9)
+    stream = torch.cuda.Stream(device=dev)
+
+    def dev_packed(vals, bits, shape_bytes):
+        t = torch.from_numpy(np.ascontiguousarray(vals).reshape(-1).astype(np.int8)).to(dev)
+        if bits != 8:
+            t = qnn.pack_subbyte(t, bits, stream=stream)
+        return t.view(torch.uint8).view(shape_bytes)
+
+    def graph_time(fn, count, reps):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(count):
+                fn(i)
+        g.replay()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / 1e3 / (count * reps)
+
+    def layer_tensors(key, layer, wl, lid, with_x=True):
+        # without an input of its own (pipeline layers) the layer's input is not drawn
+        ld = inputs.make_layer(key, layer, wl, lid, x=None if with_x else np.zeros(1, np.int64))
+        per = 8 // layer.bits
+        t = dict(
+            w=dev_packed(ld.w, layer.bits, (layer.m, layer.k, layer.k, layer.c // per)),
+            kappa=torch.from_numpy(ld.kappa).to(dev), lam=torch.from_numpy(ld.lam).to(dev),
+            bias=torch.from_numpy(ld.bias).to(dev),
+            shifts=None if ld.shifts is None else torch.from_numpy(ld.shifts).to(dev), shift=ld.shift)
+        if with_x:
+            t["x"] = dev_packed(ld.x, layer.bits, (layer.n, layer.h, layer.w, layer.c // per))
+        return ld, t
+
+    def roof(flops, nbytes, seconds):
+        ai = flops / nbytes
+        if ai >= ridge:
+            return {"bound": "tensor", "achieved": round(flops / seconds / 1e12, 1), "peak": pk["bf16_tflops"],
+                    "unit": "TFLOP/s", "frac": round(flops / seconds / 1e12 / pk["bf16_tflops"], 4),
+                    "arith_intensity": round(ai, 1)}
+        return {"bound": "hbm", "achieved": round(nbytes / seconds / 1e9, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": round(nbytes / seconds / 1e9 / pk["hbm_gbs"], 4), "arith_intensity": round(ai, 1)}
+
+    def conv_line(config, key, layer, wl, lid, extra=None):
+        ld, t = layer_tensors(key, layer, wl, lid)
+        per = 8 // layer.bits
+        set_bytes = t["x"].numel() + layer.n * layer.oh * layer.ow * layer.m // per
+        nsets = max(2, math.ceil(2 * L2_BYTES / set_bytes))
+        xs = [t["x"].clone() for _ in range(nsets)]
+        ys = [torch.empty((layer.n, layer.oh, layer.ow, layer.m // per), dtype=torch.uint8, device=dev)
+              for _ in range(nsets)]
+        kw = dict(bias=t["bias"], shifts=t["shifts"], shift=t["shift"], bits=layer.bits, stride=layer.stride,
+                  pad=layer.pad)
+        desc = qnn.conv_desc(layer.n, layer.h, layer.w, layer.c, layer.m, layer.k, layer.k, layer.stride,
+                             layer.pad, layer.bits, t["shift"])
+        algo = qnn.conv_algo(desc)
+        ws = torch.empty(max(1, qnn.workspace_size(desc)), dtype=torch.uint8, device=dev)
+
+        def call(i):
+            qnn.conv_hwc(xs[i % nsets], t["w"], t["kappa"], t["lam"], out=ys[i % nsets], workspace=ws,
+                         stream=stream, **kw)
+
+        with torch.cuda.stream(stream):
+            for i in range(3):
+                call(i)
+        torch.cuda.synchronize(dev)
+        count = max(20, min(1000, int(2e9 / max(layer.macs, 1))))
+        t_call = graph_time(call, count, 3)
+        t_kernel = None
+        if algo == qnn.ALGO_TENSORCORE:
+            prepared = qnn.PreparedConv(t["w"], t["kappa"], t["lam"], n=layer.n, h=layer.h, wd=layer.w,
+                                        bias=t["bias"], shifts=t["shifts"], shift=t["shift"], bits=layer.bits,
+                                        stride=layer.stride, pad=layer.pad, stream=stream)
+            t_kernel = graph_time(lambda i: prepared(xs[i % nsets], out=ys[i % nsets], stream=stream), count, 3)
+        qnn.device_status(stream)
+        tk = t_kernel if t_kernel is not None else t_call
+        line = {"sweep": config, "layer": layer.name, "algo": "tensorcore" if algo == qnn.ALGO_TENSORCORE else "direct",
+                "macs": layer.macs, "gmacs_call": round(layer.macs / t_call / 1e9, 1), "us_call": round(t_call * 1e6, 3),
+                "gmacs_kernel": round(layer.macs / tk / 1e9, 1), "us_kernel": round(tk * 1e6, 3),
+                "algorithmic_bytes": layer.algorithmic_bytes(), "roofline": roof(2.0 * layer.macs, layer.algorithmic_bytes(), tk),
+                "l2": f"rotating {nsets} buffer sets"}
+        if extra:
+            line.update(extra)
+        print(json.dumps(line), flush=True)
+        return t_call
+
+    # config 1: batch 1, latency; graph-captured and plain launches
+    (key, layer, wl, lid), = inputs.single_layer_workload(inputs.WORKLOAD_SINGLE)
+    t_graph = conv_line("1", key, layer, wl, lid)
+    ld, t = layer_tensors(key, layer, wl, lid)
+    y = torch.empty((1, 16, 16, 64), dtype=torch.uint8, device=dev)
+    with torch.cuda.stream(stream):
+        for _ in range(20):
+            qnn.conv_hwc(t["x"], t["w"], t["kappa"], t["lam"], bias=t["bias"], shift=t["shift"], pad=1, out=y,
+                         stream=stream)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(200):
+            qnn.conv_hwc(t["x"], t["w"], t["kappa"], t["lam"], bias=t["bias"], shift=t["shift"], pad=1, out=y,
+                         stream=stream)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_plain = e0.elapsed_time(e1) / 1e3 / 200
+    print(json.dumps({"sweep": "1", "layer": layer.name, "us_call_graph": round(t_graph * 1e6, 3),
+                      "us_call_plain_launch": round(t_plain * 1e6, 3)}), flush=True)
+
+    # config 4: INT-4 and INT-2
+    for key, layer, wl, lid in inputs.single_layer_workload(inputs.WORKLOAD_SUBBYTE):
+        conv_line("4", key, layer, wl, lid)
+    # config 5: larger layers at batch 64
+    for key, layer, wl, lid in inputs.single_layer_workload(inputs.WORKLOAD_SWEEP):
+        conv_line("5", key, layer, wl, lid)
+    # config 3: the CIFAR-shaped network, each layer, then the whole pipeline
+    layers = inputs.cifar_layers(1024)
+    for key, layer, wl, lid in layers:
+        conv_line("3", key, layer, wl, lid)
+    run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev)
+
+
+def run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev):
+    """Config 3 end to end on the device: conv, pool, conv, pool, conv, pool, FC per step."""
+    import torch
+    from paper_1908_11263_gb300 import qnn
+    n = layers[0][1].n
+    xin = torch.from_numpy(inputs.cifar_input(n).astype(np.uint8)).to(dev)
+    tensors = [layer_tensors(key, layer, wl, lid, with_x=False)[1] for key, layer, wl, lid in layers]
+    fw, fb = inputs.cifar_fc()
+    fw, fb = torch.from_numpy(fw).to(dev), torch.from_numpy(fb).to(dev)
+    bufs = []
+    for (_, layer, _, _) in layers:
+        bufs.append(torch.empty((n, layer.oh, layer.ow, layer.m), dtype=torch.uint8, device=dev))
+        bufs.append(torch.empty((n, layer.oh // 2, layer.ow // 2, layer.m), dtype=torch.uint8, device=dev))
+    out = torch.empty((n, 10), dtype=torch.int32, device=dev)
+
+    def net(_):
+        a = xin
+        for li, (_, layer, _, _) in enumerate(layers):
+            t = tensors[li]
+            qnn.conv_hwc(a, t["w"], t["kappa"], t["lam"], bias=t["bias"], shift=t["shift"], pad=layer.pad,
+                         out=bufs[2 * li], stream=stream)
+            qnn.maxpool(bufs[2 * li], 2, 2, 8, out=bufs[2 * li + 1], stream=stream)
+            a = bufs[2 * li + 1]
+        qnn.linear(a.view(n, -1), fw, fb, out=out, stream=stream)
+
+    with torch.cuda.stream(stream):
+        net(0)
+    torch.cuda.synchronize(dev)
+    t_net = graph_time(net, 20, 5)
+    qnn.device_status(stream)
+    macs = sum(layer.macs for (_, layer, _, _) in layers) + n * 1024 * 10
+    print(json.dumps({"sweep": "3", "layer": "cifar_pipeline_n1024 (3 conv + 3 pool + FC, one graph)",
+                      "macs": macs, "gmacs_call": round(macs / t_net / 1e9, 1), "us_call": round(t_net * 1e6, 3),
+                      "images_per_s": round(n / t_net, 1)}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -434,7 +607,11 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--sweep", action="store_true", help="per-config measurement lines (workloads 1, 3, 4, 5)")
     args = ap.parse_args()
+    if args.sweep:
+        run_sweep(args)
+        return
     if args.impl == "reference":
         # the oracle runs on rank 0's host cores only; other ranks exit without work
         world = int(os.environ.get("WORLD_SIZE", "1"))
