@@ -561,6 +561,45 @@ def run_sweep(args):
     for key, layer, wl, lid in layers:
         conv_line("3", key, layer, wl, lid)
     run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev)
+    run_pool_linear(graph_time, stream, dev, pk)
+
+
+def run_pool_linear(graph_time, stream, dev, pk):
+    """qmaxpool (2x2, stride 2) and qlinear on the CIFAR network's shapes, against the HBM roof."""
+    import torch
+    from paper_1908_11263_gb300 import qnn
+    rng = np.random.default_rng(11)
+    for (n, h, w, c, bits) in ((1024, 32, 32, 32, 8), (1024, 16, 16, 32, 8), (1024, 8, 8, 64, 8),
+                               (512, 16, 16, 64, 4), (512, 16, 16, 64, 2)):
+        per = 8 // bits
+        in_bytes = n * h * w * c // per
+        out_bytes = in_bytes // 4
+        nsets = max(2, math.ceil(2 * L2_BYTES / (in_bytes + out_bytes)))
+        xs = [torch.from_numpy(rng.integers(0, 256, size=(n, h, w, c // per), dtype=np.uint8)).to(dev)
+              for _ in range(min(nsets, 4))]
+        xs = [xs[i % len(xs)].clone() for i in range(nsets)]
+        ys = [torch.empty((n, h // 2, w // 2, c // per), dtype=torch.uint8, device=dev) for _ in range(nsets)]
+        t = graph_time(lambda i: qnn.maxpool(xs[i % nsets], 2, 2, bits, out=ys[i % nsets], stream=stream), 200, 3)
+        gbs = (in_bytes + out_bytes) / t / 1e9
+        print(json.dumps({"sweep": "pool", "layer": f"qmaxpool 2x2/2 {n}x{h}x{w}x{c} INT-{bits}",
+                          "us_kernel": round(t * 1e6, 3), "algorithmic_bytes": in_bytes + out_bytes,
+                          "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": pk["hbm_gbs"],
+                                       "unit": "GB/s", "frac": round(gbs / pk["hbm_gbs"], 4)},
+                          "l2": f"rotating {nsets} buffer sets"}), flush=True)
+    n, k, m = 1024, 1024, 10
+    nsets = max(2, math.ceil(2 * L2_BYTES / (n * k + n * m * 4)))
+    xs = [torch.from_numpy(rng.integers(0, 256, size=(n, k), dtype=np.uint8)).to(dev) for _ in range(nsets)]
+    wt = torch.from_numpy(rng.integers(-128, 128, size=(m, k), dtype=np.int8)).to(dev)
+    bias = torch.from_numpy(rng.integers(-4096, 4097, size=m).astype(np.int32)).to(dev)
+    ys = [torch.empty((n, m), dtype=torch.int32, device=dev) for _ in range(nsets)]
+    t = graph_time(lambda i: qnn.linear(xs[i % nsets], wt, bias, out=ys[i % nsets], stream=stream), 200, 3)
+    nbytes = n * k + m * k + m * 4 + n * m * 4
+    gbs = nbytes / t / 1e9
+    print(json.dumps({"sweep": "linear", "layer": f"qlinear {n}x{k} -> {m} (int32 out)", "us_kernel": round(t * 1e6, 3),
+                      "macs": n * k * m, "algorithmic_bytes": nbytes,
+                      "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+                                   "frac": round(gbs / pk["hbm_gbs"], 4)},
+                      "l2": f"rotating {nsets} buffer sets"}), flush=True)
 
 
 def run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev):

@@ -1,7 +1,7 @@
 // Max-pooling on packed NHWC activations (Sec. IV-A; split over output pixels as
-// in Sec. IV-B).  One thread produces 16 output bytes (INT-8 with 16 | row bytes:
-// 128-bit loads and per-byte vmax) or one output byte (any layout, field-wise max
-// of the packed sub-byte values).  No padding, floor output size.
+// in Sec. IV-B).  One thread produces 16 output bytes (pixels of whole 16-byte
+// vectors: 128-bit loads and a field-wise vmax at any Q) or one output byte (any
+// layout).  No padding, floor output size.
 #include <cstdint>
 
 #include "internal.h"
@@ -9,10 +9,28 @@
 namespace qnn {
 namespace {
 
-__global__ void __launch_bounds__(256) maxpool_u8x16_kernel(int n, int h, int w, int c, int k, int s, int oh, int ow,
-                                                            const uint4 *x, uint4 *y)
+// Field-wise maximum of two words of packed unsigned Q-bit values.  Masking
+// keeps every field at its own bit offset, so a byte-wise comparison of the
+// masked bytes orders the fields themselves.
+template <int BITS>
+__device__ __forceinline__ uint32_t max_fields(uint32_t a, uint32_t b)
 {
-    const int vec_per_pix = c / 16;
+    if (BITS == 8) return __vmaxu4(a, b);
+    uint32_t r = 0;
+#pragma unroll
+    for (int f = 0; f < 8 / BITS; ++f) {
+        const uint32_t m = ((1u << BITS) - 1u) * 0x01010101u << (f * BITS);
+        r |= __vmaxu4(a & m, b & m);
+    }
+    return r;
+}
+
+// One thread produces one 16-byte vector of an output pixel (pixels whose bytes
+// are whole 16-byte vectors).
+template <int BITS>
+__global__ void __launch_bounds__(256) maxpool_vec_kernel(int n, int h, int w, int vec_per_pix, int k, int s, int oh,
+                                                          int ow, const uint4 *x, uint4 *y)
+{
     const long long total = static_cast<long long>(n) * oh * ow * vec_per_pix;
     const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (gid >= total) return;
@@ -26,10 +44,10 @@ __global__ void __launch_bounds__(256) maxpool_u8x16_kernel(int n, int h, int w,
         for (int j = 0; j < k; ++j) {
             const long long src = ((static_cast<long long>(b) * h + oy * s + i) * w + ox * s + j) * vec_per_pix + v;
             const uint4 t = __ldg(x + src);
-            best.x = __vmaxu4(best.x, t.x);
-            best.y = __vmaxu4(best.y, t.y);
-            best.z = __vmaxu4(best.z, t.z);
-            best.w = __vmaxu4(best.w, t.w);
+            best.x = max_fields<BITS>(best.x, t.x);
+            best.y = max_fields<BITS>(best.y, t.y);
+            best.z = max_fields<BITS>(best.z, t.z);
+            best.w = max_fields<BITS>(best.w, t.w);
         }
     y[gid] = best;
 }
@@ -73,12 +91,18 @@ cudaError_t launch_maxpool(int n, int h, int w, int c, int k, int s, int bits, c
     const int oh = (h - k) / s + 1, ow = (w - k) / s + 1;
     const long long pix = static_cast<long long>(n) * oh * ow;
     if (pix == 0) return cudaSuccess;
-    const bool vec = bits == 8 && c % 16 == 0 && (reinterpret_cast<uintptr_t>(x) % 16) == 0 &&
+    const int bytes_per_pix = c * bits / 8;
+    const bool vec = bytes_per_pix % 16 == 0 && (reinterpret_cast<uintptr_t>(x) % 16) == 0 &&
                      (reinterpret_cast<uintptr_t>(y) % 16) == 0;
     if (vec) {
-        const long long total = pix * (c / 16);
-        maxpool_u8x16_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(
-            n, h, w, c, k, s, oh, ow, reinterpret_cast<const uint4 *>(x), reinterpret_cast<uint4 *>(y));
+        const int vpp = bytes_per_pix / 16;
+        const long long total = pix * vpp;
+        const unsigned grid = static_cast<unsigned>((total + 255) / 256);
+        const uint4 *xv = reinterpret_cast<const uint4 *>(x);
+        uint4 *yv = reinterpret_cast<uint4 *>(y);
+        if (bits == 8) maxpool_vec_kernel<8><<<grid, 256, 0, st>>>(n, h, w, vpp, k, s, oh, ow, xv, yv);
+        else if (bits == 4) maxpool_vec_kernel<4><<<grid, 256, 0, st>>>(n, h, w, vpp, k, s, oh, ow, xv, yv);
+        else maxpool_vec_kernel<2><<<grid, 256, 0, st>>>(n, h, w, vpp, k, s, oh, ow, xv, yv);
     } else {
         const long long total = pix * (c * bits / 8);
         const unsigned grid = static_cast<unsigned>((total + 255) / 256);

@@ -242,7 +242,7 @@ def test_workload_cifar_pipeline():
 # ------------------------------------------------------------------ max-pool, FC, packing
 
 @pytest.mark.parametrize("bits,c,k,s", [(8, 32, 2, 2), (8, 64, 3, 2), (8, 24, 2, 2), (8, 5, 2, 1), (4, 32, 2, 2),
-                                        (2, 16, 3, 3), (4, 6, 2, 2)])
+                                        (2, 16, 3, 3), (4, 6, 2, 2), (4, 64, 2, 2), (2, 64, 3, 2), (2, 128, 2, 2)])
 def test_maxpool_parity(bits, c, k, s):
     rng = np.random.default_rng(c * k + bits)
     n, h, w = 3, 11, 9
@@ -257,7 +257,8 @@ def test_maxpool_parity(bits, c, k, s):
     np.testing.assert_array_equal(out.cpu().numpy().reshape(-1), want)
 
 
-@pytest.mark.parametrize("n,k,m", [(1024, 1024, 10), (5, 7, 3), (33, 64, 17), (1, 4, 1)])
+@pytest.mark.parametrize("n,k,m", [(1024, 1024, 10), (5, 7, 3), (33, 64, 17), (1, 4, 1), (64, 2048, 40),
+                                   (8, 4096, 64)])
 def test_linear_parity(n, k, m):
     rng = np.random.default_rng(n + k + m)
     x = rng.integers(0, 256, size=(n, k)).astype(np.uint8)
