@@ -58,6 +58,9 @@ def _load():
             lib.oracle_conv_hwc.argtypes = [i32] * 12 + [P] * 6 + [i32, P, i32]
             lib.oracle_conv_hwc_pixels.argtypes = [i32] * 12 + [P] * 6 + [i32, P, i32, P]
             lib.oracle_maxpool.argtypes = [i32] * 7 + [P, P]
+            lib.oracle_staircase.argtypes = [i64, P, i32]
+            lib.oracle_staircase.restype = ctypes.c_int32
+            lib.oracle_conv_hwc_thresholds.argtypes = [i32] * 12 + [P] * 4 + [i32]
             lib.oracle_linear.argtypes = [i32] * 3 + [P] * 4
             _lib = lib
     return _lib
@@ -132,6 +135,27 @@ def conv_hwc(x_packed, w_packed, shape, bias, kappa, lam, shifts=None, shift=0, 
                                  _ptr(kappa), _ptr(lam), _ptr(shifts), int(shift), _ptr(y), int(nthreads))
     _check(st, "conv_hwc")
     return y
+
+
+def staircase(acc, tau, bits):
+    """Staircase compression of one accumulator against one channel's thresholds (Eq. 4)."""
+    t = _c(np.asarray(tau), np.int32)
+    assert t.size == (1 << bits) - 1
+    return int(_load().oracle_staircase(int(acc), _ptr(t), bits))
+
+
+def conv_hwc_thresholds(x_packed, w_packed, shape, thresholds, nthreads=1):
+    """Full layer with staircase compression; thresholds int32 [m][2^Q - 1]."""
+    s = shape
+    oh, ow = out_size(s["h"], s["w"], s["kh"], s["kw"], s["sh"], s["sw"], s["ph"], s["pw"])
+    ny = s["n"] * oh * ow * s["m"]
+    y = np.zeros(max(1, ny * s["bits"] // 8), np.uint8)
+    t = _c(np.asarray(thresholds).reshape(s["m"], (1 << s["bits"]) - 1), np.int32)
+    st = _load().oracle_conv_hwc_thresholds(s["n"], s["h"], s["w"], s["c"], s["m"], s["kh"], s["kw"], s["sh"], s["sw"],
+                                            s["ph"], s["pw"], s["bits"], _ptr(_c(x_packed, np.uint8)),
+                                            _ptr(_c(w_packed, np.uint8)), _ptr(t), _ptr(y), int(nthreads))
+    _check(st, "oracle_conv_hwc_thresholds")
+    return y[:ny * s["bits"] // 8]
 
 
 def conv_hwc_pixels(x_packed, w_packed, shape, bias, kappa, lam, pixels, shifts=None, shift=0):

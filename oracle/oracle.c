@@ -187,6 +187,55 @@ int oracle_conv_hwc(int n, int h, int w, int c, int m, int kh, int kw, int sh, i
     return status;
 }
 
+/* Staircase compression (Sec. III-A, Eq. 4): the output is the number of the
+ * channel's 2^Q - 1 thresholds that do not exceed the accumulator.  For sorted
+ * thresholds this is the index p of the interval [tau_p, tau_p+1) holding the
+ * accumulator, counted from 0 for the lowest interval (unsigned outputs; the
+ * thresholds absorb bias and batch normalisation, per the footnote to Eq. 3). */
+int32_t oracle_staircase(int64_t acc, const int32_t *tau, int bits)
+{
+    int32_t y = 0;
+    for (int k = 0; k < (1 << bits) - 1; ++k)
+        if ((int64_t)tau[k] <= acc) ++y;
+    return y;
+}
+
+/* Full layer with staircase compression: thresholds are [m][2^Q - 1] (int32). */
+int oracle_conv_hwc_thresholds(int n, int h, int w, int c, int m, int kh, int kw, int sh, int sw, int ph, int pw,
+                               int bits, const uint8_t *x_packed, const uint8_t *w_packed, const int32_t *thresholds,
+                               uint8_t *y_packed, int nthreads)
+{
+    int oh, ow;
+    if (!valid_bits(bits)) return ORACLE_EINVAL;
+    if (!conv_shape_ok(n, h, w, c, m, kh, kw, sh, sw, ph, pw, &oh, &ow)) return ORACLE_EINVAL;
+    int64_t nx = (int64_t)n * h * w * c, nw = (int64_t)m * kh * kw * c, ny = (int64_t)n * oh * ow * m;
+    if (nx % (8 / bits) || nw % (8 / bits) || ny % (8 / bits)) return ORACLE_EINVAL;
+    const int nt = (1 << bits) - 1;
+    int32_t *x = (int32_t *)malloc(sizeof(int32_t) * (size_t)(nx ? nx : 1));
+    int32_t *wt = (int32_t *)malloc(sizeof(int32_t) * (size_t)nw);
+    int32_t *y = (int32_t *)malloc(sizeof(int32_t) * (size_t)(ny ? ny : 1));
+    if (!x || !wt || !y) { free(x); free(wt); free(y); return ORACLE_EINVAL; }
+    oracle_unpack(x_packed, nx, bits, 0, x);
+    oracle_unpack(w_packed, nw, bits, 1, wt);
+    int status = ORACLE_OK;
+    if (nthreads < 1) nthreads = 1;
+#pragma omp parallel for num_threads(nthreads) schedule(dynamic, 1)
+    for (int b = 0; b < n; ++b) {
+        const int32_t *x_img = x + (int64_t)b * h * w * c;
+        for (int oy = 0; oy < oh; ++oy)
+            for (int ox = 0; ox < ow; ++ox)
+                for (int o = 0; o < m; ++o) {
+                    int64_t acc = conv_sum(h, w, c, kh, kw, sh, sw, ph, pw, x_img, wt + (int64_t)o * kh * kw * c,
+                                           oy, ox);
+                    if (!fits_i32(acc)) status = ORACLE_EOVERFLOW;
+                    y[(((int64_t)b * oh + oy) * ow + ox) * m + o] = oracle_staircase(acc, thresholds + (int64_t)o * nt, bits);
+                }
+    }
+    if (status == ORACLE_OK) oracle_pack(y, ny, bits, y_packed);
+    free(x); free(wt); free(y);
+    return status;
+}
+
 /* Same layer, evaluated only at listed output pixels (triples n, oy, ox); writes
  * the unpacked outputs [npix][m].  Used to check very large layers one output
  * pixel at a time. */

@@ -339,3 +339,68 @@ def test_paper_benchmark_layer_mac_count():
     assert int(acc.sum()) == g["macs"]
     # the paper's own cycle counts give 13.07 MAC/cycle on 8 cores
     assert round(g["macs"] / g["table2_cycles_8cores"], 2) == 13.07
+
+
+# ------------------------------------------------------------------ staircase compression (Eq. 4)
+
+def eq4_staircase(acc, tau, bits):
+    """Eq. 4 written out: the sum over output levels p of p times the characteristic function of
+    [tau_p, tau_p+1).  Levels run 0..2^Q-1 (unsigned outputs); the lowest interval is open below
+    and the highest open above."""
+    bounds = [-float("inf")] + [int(t) for t in tau] + [float("inf")]
+    return sum(p * (1 if bounds[p] <= acc < bounds[p + 1] else 0) for p in range(1 << bits))
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+def test_staircase_is_eq4_on_sorted_thresholds(bits):
+    rng = np.random.default_rng(40 + bits)
+    for _ in range(300):
+        tau = np.sort(rng.integers(-5000, 5000, size=(1 << bits) - 1))
+        if rng.random() < 0.3:  # ties: empty intervals
+            tau[rng.integers(0, tau.size - 1)] = tau[-1]
+            tau = np.sort(tau)
+        for acc in list(rng.integers(-6000, 6000, size=8)) + [int(tau[0]), int(tau[-1]), int(tau[0]) - 1]:
+            assert oracle.staircase(int(acc), tau, bits) == eq4_staircase(int(acc), tau, bits)
+
+
+def affine_thresholds(bias, kappa, lam, shift, bits):
+    """Thresholds at which clip(floor(((acc + b) * kappa + lam) / 2^s), 0, 2^Q-1) steps up, for kappa > 0:
+    the output reaches p exactly when acc >= ceil((p * 2^s - lam) / kappa) - b."""
+    tau = []
+    for p in range(1, 1 << bits):
+        num = p * (1 << shift) - int(lam)
+        t = -((-num) // int(kappa)) - int(bias)  # ceil division
+        tau.append(min(max(t, -(1 << 31)), (1 << 31) - 1))
+    return tau
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+def test_thresholds_reproduce_affine_compression(bits):
+    """A layer compressed by thresholds derived from (bias, kappa, lambda, shift) equals the same layer
+    compressed by scaling and clipping: two formulations of Sec. III-A agree on every output."""
+    rng = np.random.default_rng(50 + bits)
+    n, h, w, c, m, k = 2, 6, 7, 16, 16, 3
+    top = (1 << bits) - 1
+    x = rng.integers(0, top + 1, size=(n, h, w, c))
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, k, k, c))
+    bias = rng.integers(-300, 300, size=m).astype(np.int32)
+    kappa = rng.integers(1, 60, size=m).astype(np.int16)
+    lam = rng.integers(-4000, 4000, size=m).astype(np.int32)
+    shift = 9
+    tau = np.array([affine_thresholds(bias[o], kappa[o], lam[o], shift, bits) for o in range(m)], np.int32)
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=k, kw=k, sh=1, sw=1, ph=1, pw=1, bits=bits)
+    xp, wp = oracle.pack(x.reshape(-1), bits), oracle.pack(wt.reshape(-1), bits)
+    got = oracle.conv_hwc_thresholds(xp, wp, shape, tau)
+    want = oracle.conv_hwc(xp, wp, shape, bias, kappa, lam, shift=shift)
+    np.testing.assert_array_equal(got, want)
+    assert len(np.unique(oracle.unpack(want, want.size * 8 // bits, bits, False))) > 2  # not all clipped
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+def test_staircase_extremes(bits):
+    n_tau = (1 << bits) - 1
+    for acc in (-(1 << 30), -1, 0, 1, (1 << 30) - 1):
+        assert oracle.staircase(acc, [(1 << 31) - 1] * n_tau, bits) == 0
+        assert oracle.staircase(acc, [-(1 << 31)] * n_tau, bits) == n_tau
+        assert oracle.staircase(acc, [acc] * n_tau, bits) == n_tau        # tau <= acc counts
+        assert oracle.staircase(acc, [acc + 1] * n_tau, bits) == 0
