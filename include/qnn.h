@@ -132,6 +132,28 @@ qnn_status qconv_hwc_prepare(const qnn_conv_desc *d, const void *w, const int32_
 qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const void *workspace,
                          size_t workspace_bytes, void *stream);
 
+/*
+ * Quantized convolution with staircase compression (Sec. III-A, Eq. 4), the
+ * paper's compression for INT-4 and INT-2 outputs:
+ *
+ *   acc[n][oy][ox][o] = as in qconv_hwc() (int32, no bias)
+ *   y[n][oy][ox][o]   = number of k in [0, 2^Q - 1) with thresholds[o][k] <= acc
+ *
+ * For thresholds sorted ascending per channel this is the index p of the
+ * interval [tau_p, tau_p+1) that holds the accumulator, counted from 0 for the
+ * lowest interval (unsigned outputs).  The thresholds absorb bias and batch
+ * normalisation (footnote to Eq. 3), so there is no bias, kappa or lambda.
+ *
+ *   x, w, y     as in qconv_hwc(); d->bits must be 4 or 2 (else QNN_EUNSUPPORTED)
+ *   thresholds  device int32 [m][2^Q - 1], 4-byte aligned (any values)
+ *   workspace, workspace_bytes: as in qconv_hwc() (qconv_hwc_workspace_size)
+ *
+ * d->shift is ignored.  Same accumulator bound and other requirements as
+ * qconv_hwc().
+ */
+qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds,
+                                void *y, void *workspace, size_t workspace_bytes, void *stream);
+
 /* Which kernel qconv_hwc() would run for d: QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE;
  * negative qnn_status on invalid or unsupported descriptors. */
 int32_t qconv_hwc_algo(const qnn_conv_desc *d);

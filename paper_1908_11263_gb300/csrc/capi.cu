@@ -71,6 +71,7 @@ qnn_status check_conv(const qnn_conv_desc *d, ConvShape *s)
     if (!acc_bound_ok(static_cast<long long>(d->kh) * d->kw * d->c, d->bits)) return QNN_EUNSUPPORTED;
     s->n = d->n; s->h = d->h; s->w = d->w; s->c = d->c; s->m = d->m; s->kh = d->kh; s->kw = d->kw;
     s->sh = d->stride_h; s->sw = d->stride_w; s->ph = d->pad_h; s->pw = d->pad_w; s->bits = d->bits;
+    s->thr = 0;
     s->oh = (d->h + 2 * d->pad_h - d->kh) / d->stride_h + 1;
     s->ow = (d->w + 2 * d->pad_w - d->kw) / d->stride_w + 1;
     return QNN_OK;
@@ -233,6 +234,34 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
     if (s.n == 0) return QNN_OK;
     ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
                  d->shift, static_cast<uint8_t *>(y)};
+    return from_cuda(launch_conv_direct(s, p, cs));
+}
+
+qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds,
+                                void *y, void *workspace, size_t workspace_bytes, void *stream)
+{
+    ConvShape s;
+    qnn_status st = check_conv(d, &s);
+    if (st != QNN_OK) return st;
+    if (s.bits == 8) return QNN_EUNSUPPORTED;  // INT-8 outputs use scaling and clipping (qconv_hwc)
+    s.thr = 1;
+    if (s.n > 0 && (!x || !y)) return QNN_EINVAL;
+    if (!w || !thresholds) return QNN_EINVAL;
+    if (!aligned(x, 16) || !aligned(y, 16) || !aligned(w, 16) || !aligned(thresholds, 4)) return QNN_EALIGN;
+    TcPlan plan;
+    const int algo = choose_algo(d, s, &plan);
+    if (algo < 0) return static_cast<qnn_status>(-algo);
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), nullptr, nullptr, nullptr, nullptr,
+                 0, static_cast<uint8_t *>(y), thresholds};
+    if (algo == QNN_ALGO_TENSORCORE) {
+        st = check_workspace(plan, workspace, workspace_bytes);
+        if (st != QNN_OK) return st;
+        cudaError_t e = launch_conv_tc_prep(plan, s, p, workspace, cs);
+        if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, workspace, cs, true);
+        return from_cuda(e);
+    }
+    if (s.n == 0) return QNN_OK;
     return from_cuda(launch_conv_direct(s, p, cs));
 }
 

@@ -98,10 +98,17 @@ __global__ void __launch_bounds__(128) conv_direct_kernel(ConvShape s, ConvParam
     for (int k = 0; k < kOutPerThread; ++k) {
         if (k >= nout) break;
         const int o = o0 + k;
-        const int32_t u = acc[k] + (p.bias ? p.bias[o] : 0);
-        long long t = static_cast<long long>(u) * p.kappa[o] + p.lambda[o];
-        t >>= (p.shifts ? p.shifts[o] : p.shift);
-        const int yv = static_cast<int>(t < 0 ? 0 : (t > top ? top : t));
+        int yv;
+        if (p.thresholds) {  // staircase (Eq. 4): thresholds that do not exceed the accumulator
+            const int32_t *tau = p.thresholds + static_cast<long long>(o) * top;
+            yv = 0;
+            for (int q = 0; q < top; ++q) yv += tau[q] <= acc[k] ? 1 : 0;
+        } else {
+            const int32_t u = acc[k] + (p.bias ? p.bias[o] : 0);
+            long long t = static_cast<long long>(u) * p.kappa[o] + p.lambda[o];
+            t >>= (p.shifts ? p.shifts[o] : p.shift);
+            yv = static_cast<int>(t < 0 ? 0 : (t > top ? top : t));
+        }
         if (BITS == 8) {
             p.y[ye + k] = static_cast<uint8_t>(yv);
         } else {

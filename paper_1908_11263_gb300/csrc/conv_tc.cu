@@ -107,7 +107,10 @@ constexpr int kMaxStages = 4;
 
 // Per-channel compression constants (two records per channel, see the prep kernel).
 //   rec0 = {lam2, kappa, shift, mode}   rec1 = {beta, ulo, uhi, lambda}
-enum { kModeWide = 0, kModeClamp = 1, kModeDirect = 2 };
+enum { kModeWide = 0, kModeClamp = 1, kModeDirect = 2, kModeThreshold = 3 };
+// Staircase compression: each channel's 2^Q - 1 thresholds, stored kThrStride
+// int32 apart in the workspace and in shared memory.
+constexpr int kThrStride = 16;
 
 struct TcArgs {
     const uint8_t *x;
@@ -127,6 +130,8 @@ struct TcArgs {
     int *status;
     FastDiv fd_per_nt, fd_tpi, fd_ow, fd_w;  // n * tiles_per_img, tiles_per_img, ow, w
     int mma_warps;                            // 2: warps 12 and 15 issue alternate tiles
+    const int32_t *thr;                       // staircase thresholds in the workspace, or null
+    uint32_t off_thr;                         // their shared-memory copy
     uint32_t tap_a16[kMaxTaps];  // per tap (i, j): A offset j*copy + i*ow positions, in 16-byte units
 };
 
@@ -760,10 +765,20 @@ __device__ __noinline__ uint32_t compress64(int32_t u, int32_t kappa, int32_t la
 }
 
 // Channels whose constants need more than the direct form: raw chunk sum s ->
-// output, by the clamped 32-bit form or the 64-bit routine.
+// output, by the clamped 32-bit form, the 64-bit routine or the staircase
+// (Eq. 4: the number of the channel's thresholds that do not exceed
+// acc = s + beta; in that mode rec0.x is the shared-memory byte offset of the
+// channel's thresholds, set when the records are staged).
 __device__ __noinline__ uint32_t compress_slow(uint32_t s, int4 r0, int4 r1, uint32_t top)
 {
     const int32_t u = static_cast<int32_t>(s + static_cast<uint32_t>(r1.x));
+    if (r0.w == kModeThreshold) {
+        extern __shared__ __align__(128) uint8_t smem[];
+        const int32_t *tau = reinterpret_cast<const int32_t *>(smem + r0.x);
+        uint32_t y = 0;
+        for (uint32_t k = 0; k < top; ++k) y += tau[k] <= u ? 1u : 0u;
+        return y;
+    }
     if (r0.w == kModeClamp) {
         const int32_t uc = min(max(u, r1.y), r1.z);
         const int32_t t = (uc * r0.y + r1.w) >> r0.z;
@@ -947,12 +962,20 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
     {
         int4 *chan = reinterpret_cast<int4 *>(smem + a.off_chan);
         const int et = threadIdx.x - kConvWarps * 32, ne = kEpiWarps * 32;
-        for (int i = et; i < 2 * mp; i += ne) chan[i] = a.chan[i];
+        for (int i = et; i < 2 * mp; i += ne) {
+            int4 r = a.chan[i];
+            if (i < mp && r.w == kModeThreshold) r.x = static_cast<int>(a.off_thr) + i * 4 * kThrStride;
+            chan[i] = r;
+        }
         uint8_t *gd = reinterpret_cast<uint8_t *>(chan + 2 * mp);
         for (int gi = et; gi < mp / 16; gi += ne) {
             int all = 1;
             for (int k = 0; k < 16; ++k) all &= a.chan[gi * 16 + k].w == kModeDirect;
             gd[gi] = static_cast<uint8_t>(all);
+        }
+        if (a.thr) {
+            int32_t *ts = reinterpret_cast<int32_t *>(smem + a.off_thr);
+            for (int i = et; i < mp * kThrStride; i += ne) ts[i] = a.thr[i];
         }
         epi_barrier();
     }
@@ -1152,7 +1175,8 @@ template <int BITS>
 __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, const int32_t *bias, const int16_t *kappa,
                                                            const int32_t *lambda, const uint8_t *shifts, int shift,
                                                            int m, int mp, int kh, int kw, int c, int c_pad, int k_pad,
-                                                           int nt, int nchunks, uint16_t *wpack, int4 *chan)
+                                                           int nt, int nchunks, uint16_t *wpack, int4 *chan,
+                                                           const int32_t *thresholds, int32_t *thr_out)
 {
     pdl_trigger();
     const int lane = threadIdx.x & 31;
@@ -1190,7 +1214,18 @@ __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, con
         pos += __shfl_xor_sync(0xffffffffu, pos, d);
         neg += __shfl_xor_sync(0xffffffffu, neg, d);
     }
-    if (lane == 0) {
+    if (thresholds) {  // staircase compression: the channel's thresholds, padded channels never step up
+        for (int k = lane; k < kThrStride; k += 32)
+            thr_out[o * kThrStride + k] =
+                (o < m && k < (1 << BITS) - 1) ? thresholds[static_cast<long long>(o) * ((1 << BITS) - 1) + k] : INT32_MAX;
+    }
+    if (lane == 0 && thresholds) {
+        // the epilogue compares acc = s + beta (bias is part of the thresholds)
+        const long long off = (BITS == 8) ? -128 : 1024;
+        const uint32_t beta = 0u - static_cast<uint32_t>(off * sum) - static_cast<uint32_t>(nchunks) * kMagic;
+        chan[o] = make_int4(0, 0, 0, kModeThreshold);  // .x: threshold location, set when staged
+        chan[mp + o] = make_int4(static_cast<int32_t>(beta), 0, 0, 0);
+    } else if (lane == 0) {
         int4 r0 = make_int4(0, 0, 0, kModeDirect), r1 = make_int4(0, 0, 0, 0);
         if (o < m) {
             const long long off = (BITS == 8) ? -128 : 1024;  // staged activation = x + off
@@ -1302,7 +1337,8 @@ TcPlan plan_conv_tc(const ConvShape &s)
     const int limit = static_cast<int>(((1ll << 22) / max_prod) / 16);  // MMAs per exact chunk
     p.limit_mmas = limit;
     const int mp = p.n_ntiles * p.nt;
-    const uint32_t chan_bytes = round_up(mp * 32 + mp / 16, 16);
+    const uint32_t thr_bytes = s.thr ? static_cast<uint32_t>(mp) * 4 * kThrStride : 0;
+    const uint32_t chan_bytes = round_up(mp * 32 + mp / 16, 16) + thr_bytes;
     p.raw_stages = 2;
     for (int resident = 1; resident >= 0 && !p.cs; --resident) {
         if (resident && p.b_bytes > 120u * 1024u) continue;
@@ -1372,7 +1408,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
     p.tiles_per_img = static_cast<int>((static_cast<long long>(s.oh) * s.ow + kTileM - 1) / kTileM);
     p.total_tiles = static_cast<long long>(p.n_ntiles) * s.n * p.tiles_per_img;
     if (p.total_tiles >= (1ll << 31)) return p;
-    p.workspace_bytes = chan_offset(p) + static_cast<size_t>(mp) * 32;
+    p.workspace_bytes = chan_offset(p) + static_cast<size_t>(mp) * (32 + 4 * kThrStride);
     p.ok = true;
     return p;
 }
@@ -1383,10 +1419,11 @@ cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const Co
     uint16_t *wpack = static_cast<uint16_t *>(workspace);
     int4 *chan = reinterpret_cast<int4 *>(static_cast<uint8_t *>(workspace) + chan_offset(plan));
     const int mp = plan.n_ntiles * plan.nt;
+    int32_t *thr = reinterpret_cast<int32_t *>(chan + 2 * mp);
 #define QNN_PREP(B)                                                                                              \
     conv_tc_prep_kernel<B><<<(mp + 7) / 8, 256, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, \
                                                          mp, s.kh, s.kw, s.c, plan.c_pad, plan.k_pad, plan.nt,   \
-                                                         plan.nchunks, wpack, chan)
+                                                         plan.nchunks, wpack, chan, p.thresholds, thr)
     switch (s.bits) {
         case 8: QNN_PREP(8); break;
         case 4: QNN_PREP(4); break;
@@ -1405,6 +1442,8 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.y = y;
     a.wpack = static_cast<const uint8_t *>(workspace);
     a.chan = reinterpret_cast<const int4 *>(static_cast<const uint8_t *>(workspace) + chan_offset(plan));
+    a.thr = s.thr ? reinterpret_cast<const int32_t *>(a.chan + 2 * plan.n_ntiles * plan.nt) : nullptr;
+    a.off_thr = plan.off_chan + round_up(static_cast<uint32_t>(plan.n_ntiles * plan.nt) * 32 + plan.n_ntiles * plan.nt / 16, 16);
     a.n = s.n; a.h = s.h; a.w = s.w; a.c = s.c; a.m = s.m; a.kh = s.kh; a.kw = s.kw;
     a.ph = s.ph; a.pw = s.pw; a.oh = s.oh; a.ow = s.ow;
     a.c_pad = plan.c_pad; a.cs = plan.cs; a.nslab = plan.nslab;

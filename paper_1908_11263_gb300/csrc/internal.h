@@ -9,6 +9,7 @@ namespace qnn {
 
 struct ConvShape {
     int n, h, w, c, m, kh, kw, sh, sw, ph, pw, bits, oh, ow;
+    int thr;  // staircase compression (thresholds) instead of scaling and clipping
 };
 
 struct ConvParams {
@@ -20,6 +21,7 @@ struct ConvParams {
     const uint8_t *shifts;  // may be null
     int shift;
     uint8_t *y;
+    const int32_t *thresholds;  // [m][2^Q - 1] for staircase compression, else null
 };
 
 // ---- CUDA-core convolution (any stride / padding) -- conv_direct.cu

@@ -26,7 +26,7 @@ ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
             "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
-            "qnn_selftest_wait_timeout")
+            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds")
 
 
 class QnnError(RuntimeError):
@@ -72,6 +72,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_run.restype = I32
         lib.qconv_hwc_algo.argtypes = [DP]
         lib.qconv_hwc_noalloc.argtypes = [DP, P, P, P, P, P, P, P, P]
+        lib.qconv_hwc_thresholds.argtypes = [DP, P, P, P, P, P, SZ, P]
+        lib.qconv_hwc_thresholds.restype = I32
         lib.qconv_hwc_noalloc.restype = I32
         lib.qconv_hwc_algo.restype = I32
         lib.qlinear.argtypes = [I32, I32, I32, P, P, P, P, P]
@@ -191,6 +193,39 @@ def conv_hwc(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, strid
     st = load().qconv_hwc(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(bias), _ptr(kappa), _ptr(lam), _ptr(shifts),
                           _ptr(out), _ptr(workspace), ctypes.c_size_t(nbytes), _stream(stream))
     _check(st, "qconv_hwc")
+    return out
+
+
+def conv_hwc_thresholds(x, w, thresholds, *, bits, stride=1, pad=0, algo=ALGO_AUTO, out=None, workspace=None,
+                        stream=None):
+    """Quantized HWC convolution with staircase compression (qconv_hwc_thresholds): INT-4 or INT-2
+    outputs equal to the number of each channel's thresholds (int32 [m][2^Q - 1]) not above the
+    accumulator; returns uint8 [n, oh, ow, m*Q/8]."""
+    _dev(x, torch.uint8, "x")
+    _dev(w, (torch.int8, torch.uint8), "w")
+    _dev(thresholds, torch.int32, "thresholds")
+    per = 8 // bits
+    n, h, wd, cb = x.shape
+    m, kh, kw, cb2 = w.shape
+    if cb != cb2:
+        raise ValueError("x and w disagree on the channel count")
+    if tuple(thresholds.shape) != (m, (1 << bits) - 1):
+        raise ValueError(f"thresholds must have shape {(m, (1 << bits) - 1)}")
+    desc = conv_desc(n, h, wd, cb * per, m, kh, kw, stride, pad, bits, 0, algo)
+    oh = (h + 2 * desc.pad_h - kh) // desc.stride_h + 1
+    ow = (wd + 2 * desc.pad_w - kw) // desc.stride_w + 1
+    if out is None:
+        out = torch.empty((n, oh, ow, m // per), dtype=torch.uint8, device=x.device)
+    else:
+        _dev(out, torch.uint8, "out")
+    nbytes = workspace_size(desc)
+    if workspace is None:
+        workspace = _workspace(nbytes, x.device, stream)
+    elif workspace.numel() < nbytes:
+        raise ValueError("workspace too small")
+    st = load().qconv_hwc_thresholds(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(thresholds), _ptr(out),
+                                     _ptr(workspace), ctypes.c_size_t(nbytes), _stream(stream))
+    _check(st, "qconv_hwc_thresholds")
     return out
 
 
