@@ -321,10 +321,22 @@ __device__ __forceinline__ uint4 load_cvt(const uint8_t *p, bool ok, bool vec, c
     const uint32_t padv = pad_half2<BITS>();
     uint4 v = make_uint4(padv, padv, padv, padv);
     if (ok) {
-        if (!vec) v = cvt_generic<BITS>(row, e0, c0, c);
-        else if (BITS == 8) v = cvt_u8x8(*reinterpret_cast<const uint2 *>(p));
-        else if (BITS == 4) v = cvt_u4x8(*reinterpret_cast<const uint32_t *>(p));
-        else v = cvt_u2x8(*reinterpret_cast<const uint16_t *>(p));
+        if (!vec && BITS == 8) {
+            // C not a multiple of 8: the group's channels byte by byte (zero past C;
+            // padded channels meet zero weights)
+            uint32_t b[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) b[k] = c0 + k < c ? row[e0 + c0 + k] : 0u;
+            v = cvt_u8x8(make_uint2(b[0] | b[1] << 8 | b[2] << 16 | b[3] << 24, b[4] | b[5] << 8 | b[6] << 16 | b[7] << 24));
+        } else if (!vec) {
+            v = cvt_generic<BITS>(row, e0, c0, c);
+        } else if (BITS == 8) {
+            v = cvt_u8x8(*reinterpret_cast<const uint2 *>(p));
+        } else if (BITS == 4) {
+            v = cvt_u4x8(*reinterpret_cast<const uint32_t *>(p));
+        } else {
+            v = cvt_u2x8(*reinterpret_cast<const uint16_t *>(p));
+        }
     }
     return v;
 }
@@ -391,6 +403,8 @@ __device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *ra
         const int gq = fdiv(ci, a.fd_w);
         const int x = ci - gq * a.w;
         const int c0 = slab * a.cs + gq * 8;
+        // a group wholly past C keeps the encoded zero written at kernel start
+        if (c0 >= a.c) continue;
         // copies j in [jlo, jhi] hold this pixel (their column x + pw - j lies in [0, ow))
         const int jlo = max(0, x + a.pw - a.ow + 1), jhi = min(a.kw - 1, x + a.pw);
         bool pj[5];
