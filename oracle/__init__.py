@@ -58,6 +58,7 @@ def _load():
             lib.oracle_conv_hwc.argtypes = [i32] * 12 + [P] * 6 + [i32, P, i32]
             lib.oracle_conv_hwc_pixels.argtypes = [i32] * 12 + [P] * 6 + [i32, P, i32, P]
             lib.oracle_maxpool.argtypes = [i32] * 7 + [P, P]
+            lib.oracle_conv_binary.argtypes = [i32] * 11 + [P] * 5
             lib.oracle_staircase.argtypes = [i64, P, i32]
             lib.oracle_staircase.restype = ctypes.c_int32
             lib.oracle_conv_hwc_thresholds.argtypes = [i32] * 12 + [P] * 4 + [i32]
@@ -156,6 +157,21 @@ def conv_hwc_thresholds(x_packed, w_packed, shape, thresholds, nthreads=1):
                                             _ptr(_c(w_packed, np.uint8)), _ptr(t), _ptr(y), int(nthreads))
     _check(st, "oracle_conv_hwc_thresholds")
     return y[:ny * s["bits"] // 8]
+
+
+def conv_binary(x_bits, w_bits, shape, thresholds, with_acc=False):
+    """INT-1 layer (Eq. 5): x_bits / w_bits packed 8 per byte; returns packed output bits
+    (and the int32 popcount accumulators when asked)."""
+    s = shape
+    oh, ow = out_size(s["h"], s["w"], s["kh"], s["kw"], s["sh"], s["sw"], s["ph"], s["pw"])
+    ny = s["n"] * oh * ow * s["m"]
+    y = np.zeros(max(1, ny // 8), np.uint8)
+    acc = np.zeros(max(1, ny), np.int32) if with_acc else None
+    st = _load().oracle_conv_binary(s["n"], s["h"], s["w"], s["c"], s["m"], s["kh"], s["kw"], s["sh"], s["sw"],
+                                    s["ph"], s["pw"], _ptr(_c(x_bits, np.uint8)), _ptr(_c(w_bits, np.uint8)),
+                                    _ptr(_c(np.asarray(thresholds), np.int32)), _ptr(y), _ptr(acc))
+    _check(st, "oracle_conv_binary")
+    return (y[:ny // 8], acc[:ny]) if with_acc else y[:ny // 8]
 
 
 def conv_hwc_pixels(x_packed, w_packed, shape, bias, kappa, lam, pixels, shifts=None, shift=0):

@@ -236,6 +236,45 @@ int oracle_conv_hwc_thresholds(int n, int h, int w, int c, int m, int kh, int kw
     return status;
 }
 
+/* INT-1 (Sec. III-A, Eq. 5; binary kernel of Sec. IV-A).  Values +1 / -1 are
+ * bits 1 / 0, eight per byte, element e at bit e mod 8 of byte e / 8.  The
+ * accumulator counts the ones of W xnor X over the window positions that lie
+ * inside the image (a padded position contributes neither a match nor a
+ * mismatch: zero padding of the +-1 values); the output bit is 1 when the
+ * channel's threshold does not exceed that count. */
+static int bit_at(const uint8_t *src, int64_t e) { return (src[e >> 3] >> (e & 7)) & 1; }
+
+int oracle_conv_binary(int n, int h, int w, int c, int m, int kh, int kw, int sh, int sw, int ph, int pw,
+                       const uint8_t *x_bits, const uint8_t *w_bits, const int32_t *thresholds, uint8_t *y_bits,
+                       int32_t *acc_out)
+{
+    int oh, ow;
+    if (!conv_shape_ok(n, h, w, c, m, kh, kw, sh, sw, ph, pw, &oh, &ow)) return ORACLE_EINVAL;
+    if (c % 8 || m % 8) return ORACLE_EINVAL;
+    int64_t ny = (int64_t)n * oh * ow * m;
+    memset(y_bits, 0, (size_t)(ny / 8));
+    for (int b = 0; b < n; ++b)
+        for (int oy = 0; oy < oh; ++oy)
+            for (int ox = 0; ox < ow; ++ox)
+                for (int o = 0; o < m; ++o) {
+                    int32_t ones = 0;
+                    for (int i = 0; i < kh; ++i)
+                        for (int j = 0; j < kw; ++j) {
+                            int iy = oy * sh - ph + i, ix = ox * sw - pw + j;
+                            if (iy < 0 || iy >= h || ix < 0 || ix >= w) continue;
+                            for (int ch = 0; ch < c; ++ch) {
+                                int xb = bit_at(x_bits, (((int64_t)b * h + iy) * w + ix) * c + ch);
+                                int wb = bit_at(w_bits, (((int64_t)o * kh + i) * kw + j) * c + ch);
+                                ones += (xb == wb);  /* xnor */
+                            }
+                        }
+                    int64_t e = (((int64_t)b * oh + oy) * ow + ox) * m + o;
+                    if (acc_out) acc_out[e] = ones;
+                    if (thresholds[o] <= ones) y_bits[e >> 3] |= (uint8_t)(1u << (e & 7));
+                }
+    return ORACLE_OK;
+}
+
 /* Same layer, evaluated only at listed output pixels (triples n, oy, ox); writes
  * the unpacked outputs [npix][m].  Used to check very large layers one output
  * pixel at a time. */

@@ -404,3 +404,51 @@ def test_staircase_extremes(bits):
         assert oracle.staircase(acc, [-(1 << 31)] * n_tau, bits) == n_tau
         assert oracle.staircase(acc, [acc] * n_tau, bits) == n_tau        # tau <= acc counts
         assert oracle.staircase(acc, [acc + 1] * n_tau, bits) == 0
+
+
+# ------------------------------------------------------------------ INT-1 (Eq. 5)
+
+def bits_pack(v01):
+    """Pack 0/1 values eight per byte, element e at bit e mod 8 of byte e / 8."""
+    return np.packbits(np.asarray(v01, np.uint8).reshape(-1), bitorder="little")
+
+
+def test_binary_popcount_equals_pm1_dot_product():
+    """popcount(W xnor X) over the in-image window equals (S + K_valid) / 2, where S is the +-1 dot
+    product with zero padding and K_valid the number of in-image taps times C (torch conv2d, float64)."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(61)
+    for (n, h, w, c, m, k, s, p) in [(2, 7, 9, 16, 8, 3, 1, 1), (1, 8, 8, 8, 16, 5, 2, 2), (3, 5, 6, 24, 8, 1, 1, 0),
+                                     (1, 6, 6, 32, 8, 3, 2, 0)]:
+        xb = rng.integers(0, 2, size=(n, h, w, c))
+        wb = rng.integers(0, 2, size=(m, k, k, c))
+        shape = dict(n=n, h=h, w=w, c=c, m=m, kh=k, kw=k, sh=s, sw=s, ph=p, pw=p)
+        _, acc = oracle.conv_binary(bits_pack(xb), bits_pack(wb), shape, np.zeros(m, np.int32), with_acc=True)
+        xt = torch.from_numpy((2.0 * xb - 1).transpose(0, 3, 1, 2)).double()
+        wt = torch.from_numpy((2.0 * wb - 1).transpose(0, 3, 1, 2)).double()
+        sdot = torch.nn.functional.conv2d(xt, wt, stride=s, padding=p)
+        kvalid = torch.nn.functional.conv2d(torch.ones_like(xt), torch.ones_like(wt), stride=s, padding=p)
+        want = ((sdot + kvalid) / 2).permute(0, 2, 3, 1).numpy().reshape(-1)
+        np.testing.assert_array_equal(acc, want.astype(np.int64))
+
+
+def test_binary_threshold_and_bit_order():
+    rng = np.random.default_rng(62)
+    n, h, w, c, m, k = 2, 5, 5, 16, 16, 3
+    xb = rng.integers(0, 2, size=(n, h, w, c))
+    wb = rng.integers(0, 2, size=(m, k, k, c))
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=k, kw=k, sh=1, sw=1, ph=1, pw=1)
+    tau = rng.integers(40, 100, size=m).astype(np.int32)
+    y, acc = oracle.conv_binary(bits_pack(xb), bits_pack(wb), shape, tau, with_acc=True)
+    want = (acc.reshape(-1, m) >= tau).astype(np.uint8).reshape(-1)
+    np.testing.assert_array_equal(np.unpackbits(y, bitorder="little"), want)
+    # all +1 everywhere: every in-image tap matches; the corner pixel sees 4 of 9 taps
+    ones = np.ones((1, 4, 4, 8), np.int64)
+    shape1 = dict(n=1, h=4, w=4, c=8, m=8, kh=3, kw=3, sh=1, sw=1, ph=1, pw=1)
+    _, a1 = oracle.conv_binary(bits_pack(ones), bits_pack(np.ones((8, 3, 3, 8))), shape1, np.zeros(8, np.int32),
+                               with_acc=True)
+    assert a1.reshape(4, 4, 8)[0, 0, 0] == 4 * 8 and a1.reshape(4, 4, 8)[1, 1, 0] == 9 * 8
+    # weights the complement of the inputs: no matches at all
+    _, a2 = oracle.conv_binary(bits_pack(ones), bits_pack(np.zeros((8, 3, 3, 8))), shape1, np.zeros(8, np.int32),
+                               with_acc=True)
+    assert np.all(a2 == 0)
