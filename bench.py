@@ -39,6 +39,9 @@ from paper_1908_11263_gb300 import inputs  # noqa: E402
 L2_BYTES = 129 * 1024 * 1024
 WORKLOAD = "conv3x3_16x16x32_to_64_int8_n512"
 INT8_IMMA_TOPS = 151.6
+# 32-bit population counts per second on this GPU (all SMs; measured, 15.1 per SM per cycle at
+# 2070 MHz): the ALU roof of the INT-1 convolution, 32 binary MACs per count
+POPC_TPS = 4.77
 METRIC = "qconv_hwc GMAC/s (16x16x32 -> 64, 3x3, stride 1, pad 1, INT-8, batch 512)"
 
 
@@ -562,6 +565,32 @@ def run_sweep(args):
         conv_line("3", key, layer, wl, lid)
     run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev)
     run_pool_linear(graph_time, stream, dev, pk)
+    run_binary(graph_time, stream, dev)
+
+
+def run_binary(graph_time, stream, dev):
+    """INT-1 (XNOR / popcount) convolution on the benchmark layer's shape, against the popcount roof."""
+    import torch
+    from paper_1908_11263_gb300 import qnn
+    rng = np.random.default_rng(12)
+    n, h, w, c, m, k = 512, 16, 16, 32, 64, 3
+    xbytes, ybytes = n * h * w * c // 8, n * h * w * m // 8
+    nsets = max(2, math.ceil(2 * L2_BYTES / (xbytes + ybytes)))
+    xs = [torch.from_numpy(rng.integers(0, 256, size=(n, h, w, c // 8), dtype=np.uint8)).to(dev) for _ in range(nsets)]
+    wt = torch.from_numpy(rng.integers(0, 256, size=(m, k, k, c // 8), dtype=np.uint8)).to(dev)
+    tau = torch.full((m,), k * k * c // 2, dtype=torch.int32, device=dev)
+    ys = [torch.empty((n, h, w, m // 8), dtype=torch.uint8, device=dev) for _ in range(nsets)]
+    t = graph_time(lambda i: qnn.conv_binary(xs[i % nsets], wt, tau, pad=1, out=ys[i % nsets], stream=stream), 200, 3)
+    qnn.device_status(stream)
+    macs = n * h * w * m * k * k * c
+    achieved = macs / t / 1e12
+    peak = POPC_TPS * 32
+    print(json.dumps({"sweep": "int1", "layer": "binary conv3x3_16x16x32_to_64 n512 (XNOR/popcount)",
+                      "macs": macs, "us_kernel": round(t * 1e6, 3), "gmacs_kernel": round(macs / t / 1e9, 1),
+                      "roofline": {"bound": "alu", "achieved": round(achieved, 2), "peak": round(peak, 1),
+                                   "unit": "T binary MAC/s", "frac": round(achieved / peak, 4),
+                                   "peak_source": "measured popc rate x 32 bits per count"},
+                      "l2": f"rotating {nsets} buffer sets"}), flush=True)
 
 
 def run_pool_linear(graph_time, stream, dev, pk):

@@ -154,6 +154,28 @@ qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const v
 qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds,
                                 void *y, void *workspace, size_t workspace_bytes, void *stream);
 
+/*
+ * INT-1 convolution (Sec. III-A, Eq. 5; binary kernel of Sec. IV-A).  Values
+ * +1 / -1 are bits 1 / 0, eight per byte, element e at bit e mod 8 of byte e / 8
+ * (the sub-byte order above with Q = 1).
+ *
+ *   acc[n][oy][ox][o] = number of (i, j, ch) with the input pixel inside the
+ *                       image and bit(w[o][i][j][ch]) == bit(x[n][iy][ix][ch])
+ *                       (popcount of W xnor X; padding contributes nothing)
+ *   y[n][oy][ox][o]   = 1 if thresholds[o] <= acc, else 0
+ *
+ *   d           d->bits must be 1; c and m multiples of 8; d->shift and d->algo ignored
+ *   x           device, NHWC bits [n][h][w][c / 8 bytes]
+ *   w           device, [m][kh][kw][c / 8 bytes]
+ *   thresholds  device int32 [m], 4-byte aligned
+ *   y           device, NHWC bits [n][oh][ow][m / 8 bytes]
+ *
+ * Runs on CUDA cores (XNOR and population count).  QNN_EUNSUPPORTED when bits
+ * is not 1 or c, m are not multiples of 8.
+ */
+qnn_status qconv_hwc_binary(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds,
+                            void *y, void *stream);
+
 /* Which kernel qconv_hwc() would run for d: QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE;
  * negative qnn_status on invalid or unsupported descriptors. */
 int32_t qconv_hwc_algo(const qnn_conv_desc *d);

@@ -265,6 +265,26 @@ qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const voi
     return from_cuda(launch_conv_direct(s, p, cs));
 }
 
+qnn_status qconv_hwc_binary(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds, void *y,
+                            void *stream)
+{
+    if (!d || d->struct_size != sizeof(qnn_conv_desc)) return QNN_EINVAL;
+    if (d->n < 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->m <= 0 || d->kh <= 0 || d->kw <= 0) return QNN_EINVAL;
+    if (d->stride_h <= 0 || d->stride_w <= 0 || d->pad_h < 0 || d->pad_w < 0) return QNN_EINVAL;
+    if (d->h + 2 * d->pad_h < d->kh || d->w + 2 * d->pad_w < d->kw) return QNN_EINVAL;
+    if (d->bits != 1 || d->c % 8 || d->m % 8) return QNN_EUNSUPPORTED;
+    if (static_cast<long long>(d->kh) * d->kw * d->c >= (1ll << 31)) return QNN_EUNSUPPORTED;
+    if (!w || !thresholds || (d->n > 0 && (!x || !y))) return QNN_EINVAL;
+    if (!aligned(thresholds, 4)) return QNN_EALIGN;
+    ConvShape s{};
+    s.n = d->n; s.h = d->h; s.w = d->w; s.c = d->c; s.m = d->m; s.kh = d->kh; s.kw = d->kw;
+    s.sh = d->stride_h; s.sw = d->stride_w; s.ph = d->pad_h; s.pw = d->pad_w; s.bits = 1;
+    s.oh = (d->h + 2 * d->pad_h - d->kh) / d->stride_h + 1;
+    s.ow = (d->w + 2 * d->pad_w - d->kw) / d->stride_w + 1;
+    return from_cuda(launch_conv_binary(s, static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), thresholds,
+                                        static_cast<uint8_t *>(y), static_cast<cudaStream_t>(stream)));
+}
+
 qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
                              const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y,
                              void *stream)

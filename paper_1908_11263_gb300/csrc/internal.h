@@ -24,6 +24,10 @@ struct ConvParams {
     const int32_t *thresholds;  // [m][2^Q - 1] for staircase compression, else null
 };
 
+// ---- INT-1 convolution (XNOR / popcount, CUDA cores) -- conv_binary.cu
+cudaError_t launch_conv_binary(const ConvShape &s, const uint8_t *x, const uint8_t *w, const int32_t *thr, uint8_t *y,
+                               cudaStream_t st);
+
 // ---- CUDA-core convolution (any stride / padding) -- conv_direct.cu
 cudaError_t launch_conv_direct(const ConvShape &s, const ConvParams &p, cudaStream_t st);
 

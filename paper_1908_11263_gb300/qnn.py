@@ -26,7 +26,7 @@ ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
             "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
-            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds")
+            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary")
 
 
 class QnnError(RuntimeError):
@@ -73,6 +73,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_algo.argtypes = [DP]
         lib.qconv_hwc_noalloc.argtypes = [DP, P, P, P, P, P, P, P, P]
         lib.qconv_hwc_thresholds.argtypes = [DP, P, P, P, P, P, SZ, P]
+        lib.qconv_hwc_binary.argtypes = [DP, P, P, P, P, P]
+        lib.qconv_hwc_binary.restype = I32
         lib.qconv_hwc_thresholds.restype = I32
         lib.qconv_hwc_noalloc.restype = I32
         lib.qconv_hwc_algo.restype = I32
@@ -226,6 +228,28 @@ def conv_hwc_thresholds(x, w, thresholds, *, bits, stride=1, pad=0, algo=ALGO_AU
     st = load().qconv_hwc_thresholds(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(thresholds), _ptr(out),
                                      _ptr(workspace), ctypes.c_size_t(nbytes), _stream(stream))
     _check(st, "qconv_hwc_thresholds")
+    return out
+
+
+def conv_binary(x, w, thresholds, *, stride=1, pad=0, out=None, stream=None):
+    """INT-1 convolution (qconv_hwc_binary): x uint8 [n, h, w, c/8], w uint8 [m, kh, kw, c/8] (bits,
+    +1 = 1), thresholds int32 [m]; returns uint8 [n, oh, ow, m/8] output bits."""
+    _dev(x, torch.uint8, "x")
+    _dev(w, torch.uint8, "w")
+    _dev(thresholds, torch.int32, "thresholds")
+    n, h, wd, cb = x.shape
+    m, kh, kw, cb2 = w.shape
+    if cb != cb2:
+        raise ValueError("x and w disagree on the channel count")
+    desc = conv_desc(n, h, wd, cb * 8, m, kh, kw, stride, pad, 1, 0, ALGO_AUTO)
+    oh = (h + 2 * desc.pad_h - kh) // desc.stride_h + 1
+    ow = (wd + 2 * desc.pad_w - kw) // desc.stride_w + 1
+    if out is None:
+        out = torch.empty((n, oh, ow, m // 8), dtype=torch.uint8, device=x.device)
+    else:
+        _dev(out, torch.uint8, "out")
+    _check(load().qconv_hwc_binary(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(thresholds), _ptr(out), _stream(stream)),
+           "qconv_hwc_binary")
     return out
 
 
