@@ -125,7 +125,7 @@ struct TcArgs {
     int stages, raw_stages, b_stages, b_resident;
     int mmas_per_tile, chunk_mmas, nchunks, grp_chunks, ngroups, nsg;
     uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, chunk_stride;
-    uint32_t off_raw, off_stages, off_chan, off_bar;
+    uint32_t off_raw, off_stages, off_chan, off_bar, off_rec;
     uint32_t tmem_cols;
     int *status;
     FastDiv fd_per_nt, fd_tpi, fd_ow, fd_w;  // n * tiles_per_img, tiles_per_img, ow, w
@@ -351,8 +351,12 @@ __device__ __forceinline__ void store_copies(uint8_t *dst, uint32_t jstep, const
         if (pj[j]) *reinterpret_cast<uint4 *>(dst + j * jstep) = v;
 }
 
-// Rows rp, rp + nph, ... < rows of one column item: four rows per pass (their
-// loads in flight together), then the remaining rows one at a time.
+// Rows rp, rp + nph, ... < rows of one column item, kRowsPerPass rows per pass:
+// all of a pass's loads are in flight together before its stores, and rows
+// past the window are predicated off.  The benchmark-shaped tiles (ten staged
+// rows, two row phases) take a single pass.
+constexpr int kRowsPerPass = 6;
+
 template <int BITS, int NJ>
 __device__ __forceinline__ void convert_rows(const uint8_t *src, uint8_t *dst, int rp, int nph, int rows, int r_lo,
                                              int r_hi, bool has_data, bool vec, uint32_t row_bytes, uint32_t row_out,
@@ -361,26 +365,19 @@ __device__ __forceinline__ void convert_rows(const uint8_t *src, uint8_t *dst, i
 {
     // src / dst point at row rp; src is only dereferenced for rows inside the image
     const uint32_t src_step = row_bytes * nph, dst_step = row_out * nph;
-    int r = rp;
-    for (; r + 3 * nph < rows; r += 4 * nph) {
-        uint4 v[4];
+    for (int r = rp; r < rows; r += kRowsPerPass * nph) {
+        uint4 v[kRowsPerPass];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < kRowsPerPass; ++u) {
             const int rr = r + u * nph;
-            const bool ok = rr >= r_lo && rr < r_hi && has_data;
+            const bool ok = rr < rows && rr >= r_lo && rr < r_hi && has_data;
             v[u] = load_cvt<BITS>(src + u * src_step, ok, vec, raw + (rr - r_lo) * row_bytes, e0, c0, c);
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) store_copies<NJ>(dst + u * dst_step, jstep, pj, v[u]);
-        src += 4 * src_step;
-        dst += 4 * dst_step;
-    }
-    for (; r < rows; r += nph) {
-        const bool ok = r >= r_lo && r < r_hi && has_data;
-        const uint4 v = load_cvt<BITS>(src, ok, vec, raw + (r - r_lo) * row_bytes, e0, c0, c);
-        store_copies<NJ>(dst, jstep, pj, v);
-        src += src_step;
-        dst += dst_step;
+        for (int u = 0; u < kRowsPerPass; ++u)
+            if (r + u * nph < rows) store_copies<NJ>(dst + u * dst_step, jstep, pj, v[u]);
+        src += kRowsPerPass * src_step;
+        dst += kRowsPerPass * dst_step;
     }
 }
 
@@ -447,10 +444,14 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
     int rs = 0, stage = 0;
     uint32_t r_ph = 0, a_ph = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
-        const TileGeo g = tile_geo(a, t);
-        const uint32_t info = static_cast<uint32_t>(g.d0) | (nt_run_starts(a, t) ? kInfoRunStart : 0u) |
-                              (nt_run_ends(a, t) ? kInfoRunEnd : 0u);
         if (!warp_wait(&raw_full[rs], r_ph, a.status)) return;
+        // the tile's row window and stage word, from the loader (released with raw_full)
+        const int4 rec = *reinterpret_cast<const int4 *>(smem + a.off_rec + rs * 16);
+        TileGeo g;
+        g.rows = rec.x;
+        g.r_lo = rec.y;
+        g.r_hi = rec.z;
+        const uint32_t info = static_cast<uint32_t>(rec.w);
         const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         for (int slab = 0; slab < a.nslab; ++slab) {
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
@@ -505,7 +506,15 @@ __device__ __forceinline__ void raw_loader_role(const TcArgs &a, uint8_t *smem, 
     int issued = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
         const TileGeo g = tile_geo(a, t);
+        const uint32_t info = static_cast<uint32_t>(g.d0) | (nt_run_starts(a, t) ? kInfoRunStart : 0u) |
+                              (nt_run_ends(a, t) ? kInfoRunEnd : 0u);
         if (!warp_wait(&raw_empty[rs], ph ^ 1u, a.status)) break;
+        // The converter takes the tile geometry from here instead of recomputing
+        // it (seven reciprocal divisions on its critical path).  Lane 0 writes it
+        // and then arrives on raw_full, which releases it.
+        if ((threadIdx.x & 31) == 0)
+            *reinterpret_cast<int4 *>(smem + a.off_rec + rs * 16) =
+                make_int4(g.rows, g.r_lo, g.r_hi, static_cast<int>(info));
         const uint32_t bytes = (g.r_hi - g.r_lo) * a.row_bytes;
         if (bytes) {
             const uint8_t *src =
@@ -1371,7 +1380,9 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     const uint32_t off_chan = off_stages + stages * stage_bytes;
                     const uint32_t off_bar = off_chan + chan_bytes;
                     const uint32_t nbars = 2 * p.raw_stages + 2 * stages + 2 * b_stages + 2 * kMaxAccGroups + 1;
-                    const uint32_t total = off_bar + nbars * 8 + 4 + 4 * kMaxStages;  // TMEM slot, stage records
+                    // TMEM slot and stage words, then one 16-byte tile record per raw stage
+                    const uint32_t off_rec = round_up(off_bar + nbars * 8 + 4 + 4 * kMaxStages, 16);
+                    const uint32_t total = off_rec + 16 * p.raw_stages;
                     if (total > static_cast<uint32_t>(kMaxSmem)) continue;
                     p.cs = cs;
                     p.nslab = p.c_pad / cs;
@@ -1385,6 +1396,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     p.off_stages = off_stages;
                     p.off_chan = off_chan;
                     p.off_bar = off_bar;
+                    p.off_rec = off_rec;
                     p.smem_bytes = total;
                     break;
                 }
@@ -1475,6 +1487,7 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.chunk_stride = plan.p_alloc * 16;
     a.off_raw = plan.off_raw; a.off_stages = plan.off_stages; a.off_chan = plan.off_chan;
     a.off_bar = plan.off_bar;
+    a.off_rec = plan.off_rec;
     a.tmem_cols = plan.tmem_cols;
     a.fd_per_nt = make_fastdiv(static_cast<uint32_t>(s.n * plan.tiles_per_img));
     a.fd_tpi = make_fastdiv(static_cast<uint32_t>(plan.tiles_per_img));

@@ -56,7 +56,7 @@ struct TcPlan {
     int ngroups;        // accumulator groups in the TMEM ring
     int nsg;            // groups per tile (more than one: running sums kept in TMEM)
     uint32_t row_bytes, raw_bytes, b_bytes, b_tile_bytes, copy_bytes, stage_bytes, smem_bytes, tmem_cols;
-    uint32_t off_raw, off_stages, off_chan, off_bar;
+    uint32_t off_raw, off_stages, off_chan, off_bar, off_rec;
     size_t workspace_bytes;
 };
 
