@@ -62,6 +62,8 @@ namespace qnn {
 namespace {
 
 constexpr int kTileM = 128;
+// Strip tiles: 16 output rows x 8 output columns (see the planner).
+constexpr int kStripRows = 16, kStripCols = 8;
 // Warp roles: converters 0-3, epilogue 4-11 (two warps per TMEM lane
 // quarter, one per column half), MMA issuer 12, input-row loader 13, filter
 // loader 14, second MMA issuer 15 (takes alternate tiles when the whole
@@ -128,14 +130,21 @@ struct TcArgs {
     uint32_t off_raw, off_stages, off_chan, off_bar, off_rec;
     uint32_t tmem_cols;
     int *status;
-    FastDiv fd_per_nt, fd_tpi, fd_ow, fd_w;  // n * tiles_per_img, tiles_per_img, ow, w
+    FastDiv fd_per_nt, fd_tpi, fd_ow, fd_w;  // n * tiles_per_img, tiles_per_img, ow, pixels per staged row
+    int strip;                                // tiles are 16 x 8 strips staged as one padded window
+    int ncb, sp;                              // strips: column blocks per image, window width (pixels)
+    int ncol_w;                               // pixels per staged row: w (row tiles) or sp (strips)
+    uint32_t a_sbo;                           // A descriptor: bytes between 8-row core-matrix groups
+    uint32_t d0_mask;                         // stage-word bits the MMA adds to the A address
+    FastDiv fd_ncb;
     int mma_warps;                            // 2: warps 12 and 15 issue alternate tiles
     const int32_t *thr;                       // staircase thresholds in the workspace, or null
     uint32_t off_thr;                         // their shared-memory copy
     uint32_t tap_a16[kMaxTaps];  // per tap (i, j): A offset j*copy + i*ow positions, in 16-byte units
 };
 
-// Geometry of one tile: 128 consecutive output pixels of image `img`.
+// Geometry of one tile: 128 consecutive output pixels of image `img` (row
+// tiles), or output rows oy_a .. oy_a + 15 by columns d0 .. d0 + 7 (strips).
 struct TileGeo {
     int nt, img, ti;
     int oy_a;   // first output row touched
@@ -153,11 +162,18 @@ __device__ __forceinline__ TileGeo tile_geo(const TcArgs &a, int t)
     const int rem = t - g.nt * per_nt;
     g.img = fdiv(rem, a.fd_tpi);
     g.ti = rem - g.img * a.tiles_per_img;
-    const int p0 = g.ti * kTileM;
-    g.oy_a = fdiv(p0, a.fd_ow);
-    g.d0 = p0 - g.oy_a * a.ow;
-    const int out_rows = min(fdiv(g.d0 + kTileM + a.ow - 1, a.fd_ow), a.oh - g.oy_a);
-    g.rows = min(a.rows_max, out_rows + a.kh - 1);
+    if (a.strip) {
+        const int rb = fdiv(g.ti, a.fd_ncb);
+        g.oy_a = rb * kStripRows;
+        g.d0 = (g.ti - rb * a.ncb) * kStripCols;
+        g.rows = min(a.rows_max, a.oh - g.oy_a + a.kh - 1);
+    } else {
+        const int p0 = g.ti * kTileM;
+        g.oy_a = fdiv(p0, a.fd_ow);
+        g.d0 = p0 - g.oy_a * a.ow;
+        const int out_rows = min(fdiv(g.d0 + kTileM + a.ow - 1, a.fd_ow), a.oh - g.oy_a);
+        g.rows = min(a.rows_max, out_rows + a.kh - 1);
+    }
     const int iy0 = g.oy_a - a.ph;
     g.r_lo = min(g.rows, max(0, -iy0));
     g.r_hi = max(g.r_lo, min(g.rows, a.h - iy0));
@@ -392,8 +408,30 @@ template <int BITS>
 __device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *raw, uint8_t *stage, const TileGeo &g,
                                               int slab, bool vec, const ConvMap &mp)
 {
-    const int ncol = a.w << a.log2_groups;
+    const int ncol = a.ncol_w << a.log2_groups;
     const int cb = a.c * BITS / 8;  // packed bytes per pixel
+    if (a.strip) {
+        // One padded window, sp pixels wide: window pixel px of row r holds input
+        // pixel (r, d0 - pw + px) at position r * sp + px, the encoded zero where
+        // that pixel lies outside the image.  Every position of the tile's rows
+        // is written, so no copy and no state from earlier tiles is involved.
+        const uint32_t row_out = static_cast<uint32_t>(a.sp) * 16;
+        const bool pone[5] = {true, false, false, false, false};
+        for (int ci = mp.ci0; ci < ncol; ci += mp.cstep) {
+            const int gq = fdiv(ci, a.fd_w);
+            const int px = ci - gq * a.sp;
+            const int c0 = slab * a.cs + gq * 8;
+            if (c0 >= a.c) continue;  // a group wholly past C keeps the encoded zero
+            const int ix = g.d0 - a.pw + px;
+            const bool col_ok = ix >= 0 && ix < a.w;
+            const int rp = mp.rp;
+            const uint8_t *src = raw + (rp - g.r_lo) * static_cast<int>(a.row_bytes) + ix * cb + c0 * BITS / 8;
+            uint8_t *dst = stage + gq * a.chunk_stride + (rp * a.sp + px) * 16;
+            convert_rows<BITS, 1>(src, dst, rp, mp.nphase, g.rows, g.r_lo, g.r_hi, col_ok, vec, a.row_bytes, row_out,
+                                  0u, pone, raw, ix * a.c, c0, a.c);
+        }
+        return;
+    }
     const uint32_t jstep = a.copy_bytes - 16;
     const uint32_t row_out = static_cast<uint32_t>(a.ow) * 16;
     for (int ci = mp.ci0; ci < ncol; ci += mp.cstep) {
@@ -433,7 +471,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
 {
     const uint32_t stages_base = smem_addr(smem + a.off_stages);
     const bool vec = (a.c % 8) == 0;
-    const ConvMap mp = conv_map(a.w << a.log2_groups);
+    const ConvMap mp = conv_map(a.ncol_w << a.log2_groups);
     // encoded zero everywhere once: padding columns are never written afterwards
     {
         const uint32_t padv = pad_half2<BITS>();
@@ -452,6 +490,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
         g.r_lo = rec.y;
         g.r_hi = rec.z;
         const uint32_t info = static_cast<uint32_t>(rec.w);
+        g.d0 = static_cast<int>(info & 0xFFFFu);
         const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         for (int slab = 0; slab < a.nslab; ++slab) {
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
@@ -611,7 +650,7 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
                                                   uint64_t *done, const volatile uint32_t *stage_info, uint32_t idesc,
                                                   int nt_cols, int sel, int nsel)
 {
-    const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
+    const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, a.a_sbo);
     const uint64_t b_tmpl = smem_desc(0, nt_cols * 16, 128);
     const uint32_t stages16 = smem_addr(smem + a.off_stages) >> 4;
     const uint32_t b16 = smem_addr(smem) >> 4;
@@ -640,7 +679,7 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
             b_ph ^= 1u;
             tc_fence_after();
         }
-        const uint32_t abase = stages16 + stage * stage16 + (info & 0xFFFFu);
+        const uint32_t abase = stages16 + stage * stage16 + (info & a.d0_mask);
         bool ok = true;
         int t0 = 0;
         for (int sg = 0; sg < nsg; ++sg) {
@@ -677,7 +716,7 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                                          uint32_t idesc, int nt_cols)
 {
     const uint32_t b_lbo = nt_cols * 16;
-    const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, 128);
+    const uint64_t a_tmpl = smem_desc(0, a.chunk_stride, a.a_sbo);
     const uint64_t b_tmpl = smem_desc(0, b_lbo, 128);
     const uint32_t stages16 = smem_addr(smem + a.off_stages) >> 4;
     const uint32_t b16 = smem_addr(smem) >> 4;
@@ -715,7 +754,7 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                 b_ph ^= 1u;
                 tc_fence_after();
             }
-            const uint32_t abase = stages16 + stage * stage16 + (info & 0xFFFFu);
+            const uint32_t abase = stages16 + stage * stage16 + (info & a.d0_mask);
             int tap = 0;
             while (tap < taps) {
                 uint32_t bbase = b16 + slab * slab_b16;
@@ -1010,9 +1049,17 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
         // Pixels past the end of the image are computed but not stored.  TMEM
         // accesses are warp-collective, so every lane executes them; only the
         // store depends on the lane's pixel.
-        const int p = g.ti * kTileM + row;
+        int p;
+        bool pix_ok;
+        if (a.strip) {  // tile row = 8 * (output row - oy_a) + (output column - d0)
+            const int oy = g.oy_a + (row >> 3), ox = g.d0 + (row & 7);
+            pix_ok = oy < a.oh && ox < a.ow;
+            p = oy * a.ow + ox;
+        } else {
+            p = g.ti * kTileM + row;
+            pix_ok = p < pix_per_img;
+        }
         const int m0 = g.nt * NT + col0;
-        const bool pix_ok = p < pix_per_img;
         uint8_t *dst_row =
             ybase + (static_cast<long long>(g.img) * pix_per_img + (pix_ok ? p : 0)) * out_row_bytes;
         for (int sg = 0; sg < nsg; ++sg) {
@@ -1345,11 +1392,38 @@ TcPlan plan_conv_tc(const ConvShape &s)
     p.c_pad = (s.c + 15) / 16 * 16;
     p.k_pad = s.kh * s.kw * p.c_pad;
     p.row_bytes = static_cast<uint32_t>(row_bytes);
-    const int out_rows = std::min((s.ow - 1 + kTileM + s.ow - 1) / s.ow, s.oh);
-    p.rows_max = out_rows + s.kh - 1;
-    // positions per copy: the staged rows, and at least everything the 128 tile rows can address
-    const int reach = (s.ow - 1) + kTileM + (s.kh - 1) * s.ow;
-    p.p_alloc = static_cast<int>(round_up(static_cast<uint32_t>(std::max(p.rows_max * s.ow, reach)), 8));
+    // A tile's 128 MMA rows are 16 groups of 8 consecutive output pixels of one
+    // row, and the A descriptor steps between groups by one fixed stride.  Row
+    // tiles take 128 consecutive pixels (groups 128 B apart) and need kw copies
+    // of the staged rows, copy j shifted by j pixels, because a tap's column
+    // shift wraps around the row ends.  Strip tiles take 16 output rows by 8
+    // columns: group g is output row oy_a + g, the stride is the staged window
+    // width, and every tap (i, j) is the offset i * sp + j into a single padded
+    // window of (16 + kh - 1) x (8 + kw - 1) pixels.  Strips need kw times fewer
+    // converter stores; they are chosen unless their count (partial strips at
+    // the right and bottom edges compute pixels that are not stored) exceeds
+    // that of row tiles by more than 15 %, or row tiles cover whole output rows
+    // of a kernel at most 3 wide exactly (ow divides 128, images hold whole
+    // tiles): there row tiles stage only the rows they need and measure ~3 %
+    // faster (3x3, 16x16 images), while strips load full input rows.
+    const long long rm_tiles = (static_cast<long long>(s.oh) * s.ow + kTileM - 1) / kTileM;
+    p.ncb = (s.ow + kStripCols - 1) / kStripCols;
+    const long long strip_tiles = static_cast<long long>(p.ncb) * ((s.oh + kStripRows - 1) / kStripRows);
+    const bool rows_exact = s.kw <= 3 && s.ow >= 16 && kTileM % s.ow == 0 && (s.oh * s.ow) % kTileM == 0;
+    p.strip = s.kw > 1 && s.ow < 16384 && !rows_exact && strip_tiles * 100 <= rm_tiles * 115;
+    if (p.strip) {
+        p.sp = kStripCols + s.kw - 1;
+        p.rows_max = std::min(kStripRows, s.oh) + s.kh - 1;
+        // the MMA addresses all 16 groups' rows, stored or not
+        p.p_alloc = static_cast<int>(round_up(static_cast<uint32_t>((kStripRows + s.kh - 1) * p.sp), 8));
+    } else {
+        p.sp = 0;
+        const int out_rows = std::min((s.ow - 1 + kTileM + s.ow - 1) / s.ow, s.oh);
+        p.rows_max = out_rows + s.kh - 1;
+        // positions per copy: the staged rows, and at least everything the 128 tile rows can address
+        const int reach = (s.ow - 1) + kTileM + (s.kh - 1) * s.ow;
+        p.p_alloc = static_cast<int>(round_up(static_cast<uint32_t>(std::max(p.rows_max * s.ow, reach)), 8));
+    }
     if (p.p_alloc * 16 >= (1 << 18)) return p;  // descriptor offset field
     p.raw_bytes = round_up(static_cast<uint32_t>(p.rows_max * row_bytes), 128);
     if (p.raw_bytes >= (1u << 20)) return p;    // single transaction count
@@ -1374,7 +1448,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
                     const uint32_t b_tile = static_cast<uint32_t>(p.nt) * cs * 2;
                     const uint32_t b_region = resident ? round_up(p.b_bytes, 128) : b_stages * b_tile;
                     const uint32_t copy_bytes = static_cast<uint32_t>(p.p_alloc) * cs * 2;
-                    const uint32_t stage_bytes = copy_bytes * s.kw;
+                    const uint32_t stage_bytes = copy_bytes * (p.strip ? 1 : s.kw);
                     const uint32_t off_raw = round_up(b_region, 128);
                     const uint32_t off_stages = off_raw + p.raw_stages * p.raw_bytes;
                     const uint32_t off_chan = off_stages + stages * stage_bytes;
@@ -1431,7 +1505,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
     p.ngroups = std::min(kMaxAccGroups, (512 - sum_cols) / (p.grp_chunks * p.nt));
     p.tmem_cols = 32;
     while (p.tmem_cols < static_cast<uint32_t>(p.ngroups * p.grp_chunks * p.nt + sum_cols)) p.tmem_cols *= 2;
-    p.tiles_per_img = static_cast<int>((static_cast<long long>(s.oh) * s.ow + kTileM - 1) / kTileM);
+    p.tiles_per_img = static_cast<int>(p.strip ? strip_tiles : rm_tiles);
     p.total_tiles = static_cast<long long>(p.n_ntiles) * s.n * p.tiles_per_img;
     if (p.total_tiles >= (1ll << 31)) return p;
     p.workspace_bytes = chan_offset(p) + static_cast<size_t>(mp) * (32 + 4 * kThrStride);
@@ -1492,12 +1566,20 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.fd_per_nt = make_fastdiv(static_cast<uint32_t>(s.n * plan.tiles_per_img));
     a.fd_tpi = make_fastdiv(static_cast<uint32_t>(plan.tiles_per_img));
     a.fd_ow = make_fastdiv(static_cast<uint32_t>(s.ow));
-    a.fd_w = make_fastdiv(static_cast<uint32_t>(s.w));
+    a.strip = plan.strip;
+    a.ncb = plan.ncb;
+    a.sp = plan.sp;
+    a.ncol_w = plan.strip ? plan.sp : s.w;
+    a.fd_w = make_fastdiv(static_cast<uint32_t>(a.ncol_w));
+    a.fd_ncb = make_fastdiv(static_cast<uint32_t>(std::max(1, plan.ncb)));
+    a.a_sbo = plan.strip ? static_cast<uint32_t>(plan.sp) * 16 : 128;
+    a.d0_mask = plan.strip ? 0u : 0xFFFFu;
     // two MMA issuers when every tile of the kernel uses the same resident filter set
     a.mma_warps = (plan.b_resident && plan.nslab == 1 && plan.n_ntiles == 1) ? 2 : 1;
     for (int i = 0; i < s.kh; ++i)
         for (int j = 0; j < s.kw; ++j)
-            a.tap_a16[i * s.kw + j] = (j * plan.copy_bytes) / 16 + static_cast<uint32_t>(i * s.ow);
+            a.tap_a16[i * s.kw + j] = plan.strip ? static_cast<uint32_t>(i * plan.sp + j)
+                                                 : (j * plan.copy_bytes) / 16 + static_cast<uint32_t>(i * s.ow);
     a.status = device_status_ptr();
     if (!a.status) return cudaErrorInvalidSymbol;
     const long long sms = device_sm_count();

@@ -46,7 +46,10 @@ struct TcPlan {
     int raw_stages;     // raw input windows in flight
     int b_stages;       // filter tiles in flight (1 when resident)
     int b_resident;     // whole filter set kept in shared memory
-    int tiles_per_img;  // ceil(oh * ow / 128)
+    int tiles_per_img;  // row tiles: ceil(oh * ow / 128); strips: ceil(oh / 16) * ceil(ow / 8)
+    int strip;          // 16 x 8 strip tiles staged as one padded window (else 128-pixel row tiles)
+    int sp;             // strips: window width in pixels (8 + kw - 1)
+    int ncb;            // strips: column blocks per image
     long long total_tiles;
     int mmas_per_tile;  // MMAs (K = 16 each) per tile
     int limit_mmas;     // most MMAs one exact fp32 accumulator chunk may take

@@ -58,6 +58,12 @@ SHAPES = [
     (1, 16, 16, 12, 16, 3, 3, (1, 1), (1, 1), 4),
     (2, 16, 16, 32, 64, 3, 3, (2, 2), (1, 1), 8),
     (1, 17, 15, 16, 32, 3, 3, (2, 1), (1, 1), 4),
+    # 16 x 8 strip tiles: a partial bottom block of rows, three and five column
+    # blocks, a 5x5 window, sub-byte inputs and two channel slabs
+    (2, 30, 16, 32, 64, 3, 3, (1, 1), (1, 1), 8),
+    (1, 16, 24, 32, 48, 5, 5, (1, 1), (2, 2), 8),
+    (1, 47, 40, 32, 32, 3, 3, (1, 1), (1, 1), 4),
+    (1, 47, 40, 64, 32, 3, 3, (1, 1), (1, 1), 2),
 ]
 
 
