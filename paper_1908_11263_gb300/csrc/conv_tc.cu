@@ -137,6 +137,7 @@ struct TcArgs {
     uint32_t a_sbo;                           // A descriptor: bytes between 8-row core-matrix groups
     uint32_t d0_mask;                         // stage-word bits the MMA adds to the A address
     FastDiv fd_ncb;
+    int conv_fast;                            // converter fast path (see ConvItem)
     int mma_warps;                            // 2: warps 12 and 15 issue alternate tiles
     const int32_t *thr;                       // staircase thresholds in the workspace, or null
     uint32_t off_thr;                         // their shared-memory copy
@@ -465,6 +466,106 @@ __device__ __forceinline__ void convert_stage(const TcArgs &a, const uint8_t *ra
     }
 }
 
+// ---------------------------------------------------------------- converter fast path
+
+// A converter thread's column item, decoded once per kernel instead of once
+// per tile.  The fast path applies when each thread owns at most one item per
+// channel slab and C is a multiple of 8: it then runs a branch-free row loop.  In isolation it converts a benchmark-shaped tile in
+// about half the cycles of convert_stage(), which serves every other shape.
+struct ConvItem {
+    bool active;        // the thread owns an item
+    int px;             // image column (row tiles) or window column (strips)
+    int c0;             // first channel of the item's group within a slab
+    uint32_t src_col;   // bytes into a raw row at slab 0: pixel and channels (row tiles), channels only (strips)
+    uint32_t dst0;      // bytes into a stage for the thread's first row rp
+    uint32_t jmask;     // row tiles: the copies j that hold the pixel; strips: 1
+};
+
+template <int BITS>
+__device__ __forceinline__ ConvItem conv_item(const TcArgs &a, const ConvMap &mp)
+{
+    ConvItem it;
+    const int ncol = a.ncol_w << a.log2_groups;
+    const int ci = mp.ci0;
+    const int gq = ci / a.ncol_w;  // once per kernel
+    const int c0 = gq * 8;
+    it.px = ci - gq * a.ncol_w;
+    it.c0 = c0;
+    it.active = ci < ncol;
+    if (a.strip) {
+        it.src_col = static_cast<uint32_t>(c0 * BITS / 8);
+        it.dst0 = static_cast<uint32_t>(gq) * a.chunk_stride + static_cast<uint32_t>(mp.rp * a.sp + it.px) * 16;
+        it.jmask = 1u;
+    } else {
+        it.src_col = static_cast<uint32_t>(it.px * (a.c * BITS / 8) + c0 * BITS / 8);
+        it.dst0 = static_cast<uint32_t>(gq) * a.chunk_stride + static_cast<uint32_t>(it.px + a.pw) * 16 +
+                  static_cast<uint32_t>(mp.rp * a.ow) * 16;
+        const int jlo = max(0, it.px + a.pw - a.ow + 1), jhi = min(a.kw - 1, it.px + a.pw);
+        it.jmask = jhi >= jlo ? ((2u << jhi) - (1u << jlo)) : 0u;
+    }
+    return it;
+}
+
+template <int BITS>
+__device__ __forceinline__ uint4 cvt_raw(const uint8_t *p)
+{
+    if (BITS == 8) return cvt_u8x8(*reinterpret_cast<const uint2 *>(p));
+    if (BITS == 4) return cvt_u4x8(*reinterpret_cast<const uint32_t *>(p));
+    return cvt_u2x8(*reinterpret_cast<const uint16_t *>(p));
+}
+
+// One tile of the thread's item: rows rp, rp + nph, ... < rows, kRowsPerPass
+// per pass with every load issued before the stores.  The values written are
+// those of convert_stage(): the staged encoding inside the image, the encoded
+// zero outside it; row tiles store the copies in jmask, strips one position.
+template <int BITS, int NJ, bool STRIP>
+__device__ __forceinline__ void convert_fast(const TcArgs &a, const uint8_t *raw, uint8_t *stage, const TileGeo &g,
+                                             const ConvItem &it, const ConvMap &mp, int slab)
+{
+    // a group wholly past C keeps the encoded zero written at kernel start
+    if (!it.active || slab * a.cs + it.c0 >= a.c) return;
+    const uint32_t padv = pad_half2<BITS>();
+    const int nph = mp.nphase;
+    const int row_bytes = static_cast<int>(a.row_bytes);
+    bool col_ok = true;
+    int col = static_cast<int>(it.src_col) + slab * a.cs * BITS / 8;
+    if (STRIP) {
+        const int ix = g.d0 - a.pw + it.px;
+        col_ok = ix >= 0 && ix < a.w;
+        col += ix * (a.c * BITS / 8);
+    }
+    const uint32_t row_out = static_cast<uint32_t>(STRIP ? a.sp : a.ow) * 16;
+    const uint32_t jstep = a.copy_bytes - 16;
+    // only dereferenced for rows inside the image and pixels inside a row
+    const uint8_t *src = raw + (mp.rp - g.r_lo) * row_bytes + col;
+    uint8_t *dst = stage + it.dst0;
+    const int src_step = row_bytes * nph;
+    const uint32_t dst_step = row_out * nph;
+    for (int r = mp.rp; r < g.rows; r += kRowsPerPass * nph) {
+        // Every load is issued: rows outside the image read the raw stage's
+        // first bytes instead, and the encoded zero is selected afterwards, so
+        // the loads go out back to back with no branch between them.
+        uint4 v[kRowsPerPass];
+#pragma unroll
+        for (int u = 0; u < kRowsPerPass; ++u) {
+            const int rr = r + u * nph;
+            const bool ok = col_ok && rr >= g.r_lo && rr < g.r_hi;
+            const uint4 x = cvt_raw<BITS>(ok ? src + u * src_step : raw);
+            v[u] = ok ? x : make_uint4(padv, padv, padv, padv);
+        }
+#pragma unroll
+        for (int u = 0; u < kRowsPerPass; ++u) {
+            if (r + u * nph < g.rows) {
+#pragma unroll
+                for (int j = 0; j < NJ; ++j)
+                    if ((it.jmask >> j) & 1u) *reinterpret_cast<uint4 *>(dst + u * dst_step + j * jstep) = v[u];
+            }
+        }
+        src += kRowsPerPass * src_step;
+        dst += kRowsPerPass * dst_step;
+    }
+}
+
 template <int BITS>
 __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
                                uint64_t *a_full, uint64_t *a_empty, volatile uint32_t *stage_info)
@@ -479,6 +580,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
         const uint32_t total = a.stages * a.stage_bytes / 16;
         for (uint32_t i = threadIdx.x; i < total; i += 128) sts128(stages_base + i * 16, pad4);
     }
+    const ConvItem item = conv_item<BITS>(a, mp);
     int rs = 0, stage = 0;
     uint32_t r_ph = 0, a_ph = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
@@ -494,7 +596,15 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
         const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         for (int slab = 0; slab < a.nslab; ++slab) {
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
-            convert_stage<BITS>(a, raw, smem + a.off_stages + stage * a.stage_bytes, g, slab, vec, mp);
+            uint8_t *st = smem + a.off_stages + stage * a.stage_bytes;
+            if (!a.conv_fast)
+                convert_stage<BITS>(a, raw, st, g, slab, vec, mp);
+            else if (a.strip)
+                convert_fast<BITS, 1, true>(a, raw, st, g, item, mp, slab);
+            else if (a.kw <= 3)
+                convert_fast<BITS, 3, false>(a, raw, st, g, item, mp, slab);
+            else
+                convert_fast<BITS, 5, false>(a, raw, st, g, item, mp, slab);
             if (threadIdx.x == 0) stage_info[stage] = info;  // released by this thread's arrive below
             fence_proxy_async_smem();
             mbar_arrive(&a_full[stage]);
@@ -1574,6 +1684,7 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.fd_ncb = make_fastdiv(static_cast<uint32_t>(std::max(1, plan.ncb)));
     a.a_sbo = plan.strip ? static_cast<uint32_t>(plan.sp) * 16 : 128;
     a.d0_mask = plan.strip ? 0u : 0xFFFFu;
+    a.conv_fast = s.c % 8 == 0 && (a.ncol_w << a.log2_groups) <= 128 && (plan.strip || s.kw <= 5);
     // two MMA issuers when every tile of the kernel uses the same resident filter set
     a.mma_warps = (plan.b_resident && plan.nslab == 1 && plan.n_ntiles == 1) ? 2 : 1;
     for (int i = 0; i < s.kh; ++i)
