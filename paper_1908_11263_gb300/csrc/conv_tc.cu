@@ -1180,6 +1180,26 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
             const uint32_t grp_addr = lane_addr + grp * grp_chunks * NT;
             const bool last = sg == nsg - 1;
             uint32_t v[CW];
+            bool drained = false;
+            if constexpr (CW == 32) {
+                if (nsg == 1 && nsub == 2) {
+                    // the whole tile in one group of two buffers: per half of
+                    // the warp's columns, both buffers' loads in flight, one wait
+#pragma unroll
+                    for (int b0 = 0; b0 < 32; b0 += 16) {
+                        uint32_t t0[16], t1[16];
+                        tmem_ld16(grp_addr + b0, t0);
+                        tmem_ld16(grp_addr + NT + b0, t1);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int k = 0; k < 16; ++k) v[b0 + k] = t0[k] + t1[k];
+                        tmem_st16_fill(grp_addr + b0, kMagic);
+                        tmem_st16_fill(grp_addr + NT + b0, kMagic);
+                    }
+                    drained = true;
+                }
+            }
+            if (!drained) {
 #pragma unroll
             for (int k = 0; k < CW; ++k) v[k] = 0;
             const int nsrc = nsub + (sg > 0 ? 1 : 0);
@@ -1198,6 +1218,7 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
                     for (int k = 0; k < BATCH; ++k) v[b0 + k] += tmp[k];
                     if (!is_sum) tmem_fill_cols<BATCH>(src + b0, kMagic);
                 }
+            }
             }
             if (!last) {
 #pragma unroll
