@@ -646,6 +646,8 @@ def run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev):
         bufs.append(torch.empty((n, layer.oh // 2, layer.ow // 2, layer.m), dtype=torch.uint8, device=dev))
     out = torch.empty((n, 10), dtype=torch.int32, device=dev)
 
+    out_fused = torch.empty_like(out)
+
     def net(_):
         a = xin
         for li, (_, layer, _, _) in enumerate(layers):
@@ -656,15 +658,29 @@ def run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev):
             a = bufs[2 * li + 1]
         qnn.linear(a.view(n, -1), fw, fb, out=out, stream=stream)
 
+    def net_fused(_):
+        # each conv + pool pair as one qconv_hwc_pool2 launch pair (prep + fused kernel)
+        a = xin
+        for li, (_, layer, _, _) in enumerate(layers):
+            t = tensors[li]
+            qnn.conv_hwc_pool2(a, t["w"], t["kappa"], t["lam"], bias=t["bias"], shift=t["shift"], pad=layer.pad,
+                               out=bufs[2 * li + 1], stream=stream)
+            a = bufs[2 * li + 1]
+        qnn.linear(a.view(n, -1), fw, fb, out=out_fused, stream=stream)
+
+    macs = sum(layer.macs for (_, layer, _, _) in layers) + n * 1024 * 10
     with torch.cuda.stream(stream):
         net(0)
+        net_fused(0)
     torch.cuda.synchronize(dev)
-    t_net = graph_time(net, 20, 5)
-    qnn.device_status(stream)
-    macs = sum(layer.macs for (_, layer, _, _) in layers) + n * 1024 * 10
-    print(json.dumps({"sweep": "3", "layer": "cifar_pipeline_n1024 (3 conv + 3 pool + FC, one graph)",
-                      "macs": macs, "gmacs_call": round(macs / t_net / 1e9, 1), "us_call": round(t_net * 1e6, 3),
-                      "images_per_s": round(n / t_net, 1)}), flush=True)
+    same = bool(torch.equal(out, out_fused))
+    for fn, name in ((net, "cifar_pipeline_n1024 (3 conv + 3 pool + FC, one graph)"),
+                     (net_fused, "cifar_pipeline_fused_n1024 (3 fused conv+pool + FC, one graph)")):
+        t_net = graph_time(fn, 20, 5)
+        qnn.device_status(stream)
+        print(json.dumps({"sweep": "3", "layer": name, "macs": macs, "gmacs_call": round(macs / t_net / 1e9, 1),
+                          "us_call": round(t_net * 1e6, 3), "images_per_s": round(n / t_net, 1),
+                          "fc_outputs_equal_unfused": same}), flush=True)
 
 
 def main():

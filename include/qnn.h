@@ -133,6 +133,27 @@ qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const v
                          size_t workspace_bytes, void *stream);
 
 /*
+ * Quantized convolution, compression and 2x2 max-pooling in one kernel: the
+ * pooling layer of Sec. IV-A (window 2, stride 2, no padding, floor output
+ * size) applied to the output of qconv_hwc(), fused into its epilogue so the
+ * full-resolution output never reaches memory:
+ *
+ *   t[n][oy][ox][o]  = y of qconv_hwc() for the same arguments
+ *   y[n][py][px][o]  = max over dy, dx in {0, 1} of t[n][2*py+dy][2*px+dx][o]
+ *                      for py < oh / 2, px < ow / 2 (integer division)
+ *
+ * Arguments are those of qconv_hwc(); y is the pooled NHWC tensor
+ * [n][oh/2][ow/2][m], packed Q-bit, 16-byte aligned.  The workspace size is
+ * qconv_hwc_workspace_size() of the same descriptor.  Runs only on the
+ * tensor-core kernel (stride 1, the shapes qconv_hwc_algo() reports as
+ * QNN_ALGO_TENSORCORE, d->algo not QNN_ALGO_DIRECT); QNN_EUNSUPPORTED
+ * otherwise, and QNN_EINVAL when oh or ow is below 2 (no pooled pixel).
+ */
+qnn_status qconv_hwc_pool2(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
+                           const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y,
+                           void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * Quantized convolution with staircase compression (Sec. III-A, Eq. 4), the
  * paper's compression for INT-4 and INT-2 outputs:
  *

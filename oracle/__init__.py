@@ -198,6 +198,16 @@ def maxpool(x_packed, n, h, w, c, k, s, bits):
     return y
 
 
+def conv_hwc_pool2(x_packed, w_packed, shape, bias, kappa, lam, shifts=None, shift=0, nthreads=1):
+    """A convolution layer followed by a 2x2, stride-2 max-pooling layer over its quantized output
+    (Sec. IV-A lists the pooling kernel beside the convolution), stated as the two layers in
+    sequence: conv_hwc, then maxpool with window 2 and stride 2 (floor output size)."""
+    y = conv_hwc(x_packed, w_packed, shape, bias, kappa, lam, shifts=shifts, shift=shift, nthreads=nthreads)
+    s = shape
+    oh, ow = out_size(s["h"], s["w"], s["kh"], s["kw"], s["sh"], s["sw"], s["ph"], s["pw"])
+    return maxpool(y, s["n"], oh, ow, s["m"], 2, 2, s["bits"])
+
+
 def linear(x, w, bias):
     """x u8 [N,K], w s8 [M,K], bias i32 [M] or None -> int32 [N,M]."""
     x = _c(x, np.uint8)

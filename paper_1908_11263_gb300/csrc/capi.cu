@@ -72,6 +72,7 @@ qnn_status check_conv(const qnn_conv_desc *d, ConvShape *s)
     s->n = d->n; s->h = d->h; s->w = d->w; s->c = d->c; s->m = d->m; s->kh = d->kh; s->kw = d->kw;
     s->sh = d->stride_h; s->sw = d->stride_w; s->ph = d->pad_h; s->pw = d->pad_w; s->bits = d->bits;
     s->thr = 0;
+    s->pool = 0;
     s->oh = (d->h + 2 * d->pad_h - d->kh) / d->stride_h + 1;
     s->ow = (d->w + 2 * d->pad_w - d->kw) / d->stride_w + 1;
     return QNN_OK;
@@ -235,6 +236,32 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
     ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
                  d->shift, static_cast<uint8_t *>(y)};
     return from_cuda(launch_conv_direct(s, p, cs));
+}
+
+qnn_status qconv_hwc_pool2(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
+                           const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y, void *workspace,
+                           size_t workspace_bytes, void *stream)
+{
+    ConvShape s;
+    qnn_status st = check_conv(d, &s);
+    if (st != QNN_OK) return st;
+    if (s.oh < 2 || s.ow < 2) return QNN_EINVAL;  // no pooled pixel
+    s.pool = 1;
+    if (s.n > 0 && (!x || !y)) return QNN_EINVAL;
+    if (!aligned(x, 16) || !aligned(y, 16)) return QNN_EALIGN;
+    TcPlan plan;
+    st = check_params(d, s, w, bias, kappa, lambda, shifts, &plan);
+    if (st != QNN_OK) return st;
+    // the fused pool runs in the tensor-core kernel only (strip tiles)
+    if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE || !plan.strip) return QNN_EUNSUPPORTED;
+    st = check_workspace(plan, workspace, workspace_bytes);
+    if (st != QNN_OK) return st;
+    cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
+                 d->shift, static_cast<uint8_t *>(y)};
+    cudaError_t e = launch_conv_tc_prep(plan, s, p, workspace, cs);
+    if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, workspace, cs, true);
+    return from_cuda(e);
 }
 
 qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds,

@@ -138,6 +138,7 @@ struct TcArgs {
     uint32_t d0_mask;                         // stage-word bits the MMA adds to the A address
     FastDiv fd_ncb;
     int conv_fast;                            // converter fast path (see ConvItem)
+    int pool, pool_oh, pool_ow;               // fused 2x2/2 max-pool and its output height, width
     int mma_warps;                            // 2: warps 12 and 15 issue alternate tiles
     const int32_t *thr;                       // staircase thresholds in the workspace, or null
     uint32_t off_thr;                         // their shared-memory copy
@@ -980,8 +981,8 @@ __device__ __forceinline__ uint32_t pack2_sat(int hi, int lo, uint32_t upper)
 // accumulator the layer can produce, and folded bias, the staging offset and
 // the accumulator pre-load into lam2, so the wrapped 32-bit value is exact.
 template <int BITS, int G>
-__device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *rec0, const int4 *rec1, bool direct,
-                                               int m_first, int valid, uint8_t *dst)
+__device__ __forceinline__ void compress_pack(const uint32_t *s, const int4 *rec0, const int4 *rec1, bool direct,
+                                              int m_first, uint32_t (&packed)[(G * BITS + 31) / 32])
 {
     int y[G];
     if (direct) {
@@ -997,7 +998,6 @@ __device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *re
     }
     constexpr int kPer = 32 / BITS;                   // results per 32-bit word
     constexpr int kWords = (G * BITS + 31) / 32;
-    uint32_t packed[kWords];
 #pragma unroll
     for (int wd = 0; wd < kWords; ++wd) {
         uint32_t t = 0;
@@ -1008,6 +1008,13 @@ __device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *re
         }
         packed[wd] = t;
     }
+}
+
+// Stores G packed Q-bit outputs (fewer when `valid` < G, at the end of M).
+template <int BITS, int G>
+__device__ __forceinline__ void store_packed(const uint32_t (&packed)[(G * BITS + 31) / 32], int valid, uint8_t *dst)
+{
+    constexpr int kWords = (G * BITS + 31) / 32;
     constexpr int kBytes = G * BITS / 8;
     if (valid >= G && (reinterpret_cast<uintptr_t>(dst) % kBytes) == 0) {
         if (kBytes == 16) *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
@@ -1020,6 +1027,15 @@ __device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *re
         for (int b = 0; b < kBytes; ++b)
             if (b < nbytes) dst[b] = static_cast<uint8_t>(packed[b / 4] >> (8 * (b % 4)));
     }
+}
+
+template <int BITS, int G>
+__device__ __forceinline__ void compress_store(const uint32_t *s, const int4 *rec0, const int4 *rec1, bool direct,
+                                               int m_first, int valid, uint8_t *dst)
+{
+    uint32_t packed[(G * BITS + 31) / 32];
+    compress_pack<BITS, G>(s, rec0, rec1, direct, m_first, packed);
+    store_packed<BITS, G>(packed, valid, dst);
 }
 
 // TMEM access in steps of 16 (or, for 8-column warps, 8) columns.
@@ -1095,7 +1111,7 @@ __device__ __forceinline__ void release_acc(uint64_t *bar)
 // back and releases the group before the compression arithmetic, so the MMA
 // warp can refill it meanwhile.  Tiles that take several groups carry their
 // running sums in TMEM.
-template <int BITS, int NT>
+template <int BITS, int NT, bool POOL>
 __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
                                               uint64_t *acc_empty)
 {
@@ -1172,6 +1188,18 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
         const int m0 = g.nt * NT + col0;
         uint8_t *dst_row =
             ybase + (static_cast<long long>(g.img) * pix_per_img + (pix_ok ? p : 0)) * out_row_bytes;
+        // Fused 2x2/2 max-pool (strip tiles): the window of pooled pixel
+        // (oy/2, ox/2) is tile rows 8*dy + dx apart, lanes L, L^1, L^8, L^9 of
+        // one warp; its top-left lane stores.  Windows that reach past the
+        // image have no pooled pixel (floor output size).
+        bool pool_store = false;
+        uint8_t *pool_row = ybase;
+        if constexpr (POOL) {
+            const int oy = g.oy_a + (row >> 3), ox = g.d0 + (row & 7);
+            pool_store = (row & 9) == 0 && (oy >> 1) < a.pool_oh && (ox >> 1) < a.pool_ow;
+            if (pool_store)
+                pool_row += ((static_cast<long long>(g.img) * a.pool_oh + (oy >> 1)) * a.pool_ow + (ox >> 1)) * out_row_bytes;
+        }
         for (int sg = 0; sg < nsg; ++sg) {
             if (!warp_wait(&acc_full[grp], (full_ph >> grp) & 1u, status)) return;
             full_ph ^= 1u << grp;
@@ -1231,7 +1259,22 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
             }
             release_acc(&acc_empty[grp]);
             if (++grp == ngroups) grp = 0;
-            if (last && pix_ok) {
+            if (POOL && last) {
+#pragma unroll
+                for (int c = 0; c < CW; c += G) {
+                    const int valid = m - (m0 + c);  // same for the whole warp: every lane shuffles
+                    if (valid > 0) {
+                        uint32_t pk[(G * BITS + 31) / 32];
+                        compress_pack<BITS, G>(v + c, rec0, rec1, gdirect[(m0 + c) >> 4] != 0, m0 + c, pk);
+#pragma unroll
+                        for (int wd = 0; wd < (G * BITS + 31) / 32; ++wd) {
+                            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 1));
+                            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 8));
+                        }
+                        if (pool_store) store_packed<BITS, G>(pk, valid, pool_row + (m0 + c) * BITS / 8);
+                    }
+                }
+            } else if (last && pix_ok) {
 #pragma unroll
                 for (int c = 0; c < CW; c += G) {
                     const int valid = m - (m0 + c);  // same for the whole warp
@@ -1244,7 +1287,9 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
     }
 }
 
-template <int BITS, int NT>
+// POOL: the fused 2x2/2 max-pool epilogue (a separate instantiation, so the
+// plain kernel carries none of its registers).
+template <int BITS, int NT, bool POOL>
 __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
 {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -1295,7 +1340,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     if (warp < kConvWarps) {
         converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty, stage_info);
     } else if (warp < kConvWarps + kEpiWarps) {
-        epilogue_role<BITS, NT>(a, smem, tmem_base, acc_full, acc_empty);
+        epilogue_role<BITS, NT, POOL>(a, smem, tmem_base, acc_full, acc_empty);
     } else if (warp == kMmaWarp || (warp == kMmaWarp2 && a.mma_warps == 2)) {
         const uint32_t idesc = idesc_f16_f32(kTileM, NT);
         const int sel = warp == kMmaWarp ? 0 : 1;
@@ -1450,13 +1495,13 @@ __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, con
     }
 }
 
-template <int BITS, int NT>
+template <int BITS, int NT, bool POOL>
 cudaError_t launch_tc(const TcArgs &args, int grid, uint32_t smem, cudaStream_t st, bool after_prep)
 {
     // the opt-in shared-memory limit is raised once per device, outside any stream capture
     static std::mutex mu;
     static bool raised[64] = {};
-    auto kern = conv_tc_kernel<BITS, NT>;
+    auto kern = conv_tc_kernel<BITS, NT, POOL>;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -1492,10 +1537,14 @@ template <int BITS>
 cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, cudaStream_t st, bool after_prep)
 {
     switch (nt) {
-        case 16: return launch_tc<BITS, 16>(args, grid, smem, st, after_prep);
-        case 32: return launch_tc<BITS, 32>(args, grid, smem, st, after_prep);
-        case 64: return launch_tc<BITS, 64>(args, grid, smem, st, after_prep);
-        case 128: return launch_tc<BITS, 128>(args, grid, smem, st, after_prep);
+        case 16: return args.pool ? launch_tc<BITS, 16, true>(args, grid, smem, st, after_prep)
+                                  : launch_tc<BITS, 16, false>(args, grid, smem, st, after_prep);
+        case 32: return args.pool ? launch_tc<BITS, 32, true>(args, grid, smem, st, after_prep)
+                                  : launch_tc<BITS, 32, false>(args, grid, smem, st, after_prep);
+        case 64: return args.pool ? launch_tc<BITS, 64, true>(args, grid, smem, st, after_prep)
+                                  : launch_tc<BITS, 64, false>(args, grid, smem, st, after_prep);
+        case 128: return args.pool ? launch_tc<BITS, 128, true>(args, grid, smem, st, after_prep)
+                                   : launch_tc<BITS, 128, false>(args, grid, smem, st, after_prep);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -1542,6 +1591,10 @@ TcPlan plan_conv_tc(const ConvShape &s)
     const long long strip_tiles = static_cast<long long>(p.ncb) * ((s.oh + kStripRows - 1) / kStripRows);
     const bool rows_exact = s.kw <= 3 && s.ow >= 16 && kTileM % s.ow == 0 && (s.oh * s.ow) % kTileM == 0;
     p.strip = s.kw > 1 && s.ow < 16384 && !rows_exact && strip_tiles * 100 <= rm_tiles * 115;
+    if (s.pool) {  // the fused pool needs each 2x2 window inside one warp: strips only
+        if (s.ow >= 16384) return p;
+        p.strip = true;
+    }
     if (p.strip) {
         p.sp = kStripCols + s.kw - 1;
         p.rows_max = std::min(kStripRows, s.oh) + s.kh - 1;
@@ -1706,6 +1759,9 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.a_sbo = plan.strip ? static_cast<uint32_t>(plan.sp) * 16 : 128;
     a.d0_mask = plan.strip ? 0u : 0xFFFFu;
     a.conv_fast = s.c % 8 == 0 && (a.ncol_w << a.log2_groups) <= 128 && (plan.strip || s.kw <= 5);
+    a.pool = s.pool;
+    a.pool_oh = s.oh / 2;
+    a.pool_ow = s.ow / 2;
     // two MMA issuers when every tile of the kernel uses the same resident filter set
     a.mma_warps = (plan.b_resident && plan.nslab == 1 && plan.n_ntiles == 1) ? 2 : 1;
     for (int i = 0; i < s.kh; ++i)

@@ -186,6 +186,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16])
         : "memory");
 }
 
+// Field-wise unsigned maximum of two words of packed Q-bit values (Q = 8, 4, 2).
+// Masking keeps every field at its own bit offset, so a byte-wise comparison
+// of the masked bytes orders the fields themselves.
+template <int BITS>
+__device__ __forceinline__ uint32_t max_fields(uint32_t a, uint32_t b)
+{
+    if (BITS == 8) return __vmaxu4(a, b);
+    uint32_t r = 0;
+#pragma unroll
+    for (int f = 0; f < 8 / BITS; ++f) {
+        const uint32_t m = ((1u << BITS) - 1u) * 0x01010101u << (f * BITS);
+        r |= __vmaxu4(a & m, b & m);
+    }
+    return r;
+}
+
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 // Writes the same 32-bit value into 16 consecutive columns of this thread's lane.

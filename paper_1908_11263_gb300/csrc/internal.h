@@ -10,6 +10,7 @@ namespace qnn {
 struct ConvShape {
     int n, h, w, c, m, kh, kw, sh, sw, ph, pw, bits, oh, ow;
     int thr;  // staircase compression (thresholds) instead of scaling and clipping
+    int pool; // 2x2 stride-2 max-pool of the compressed outputs, fused (strip tiles only)
 };
 
 struct ConvParams {

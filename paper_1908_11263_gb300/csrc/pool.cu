@@ -4,26 +4,11 @@
 // layout).  No padding, floor output size.
 #include <cstdint>
 
+#include "device.cuh"
 #include "internal.h"
 
 namespace qnn {
 namespace {
-
-// Field-wise maximum of two words of packed unsigned Q-bit values.  Masking
-// keeps every field at its own bit offset, so a byte-wise comparison of the
-// masked bytes orders the fields themselves.
-template <int BITS>
-__device__ __forceinline__ uint32_t max_fields(uint32_t a, uint32_t b)
-{
-    if (BITS == 8) return __vmaxu4(a, b);
-    uint32_t r = 0;
-#pragma unroll
-    for (int f = 0; f < 8 / BITS; ++f) {
-        const uint32_t m = ((1u << BITS) - 1u) * 0x01010101u << (f * BITS);
-        r |= __vmaxu4(a & m, b & m);
-    }
-    return r;
-}
 
 // One thread produces one 16-byte vector of an output pixel (pixels whose bytes
 // are whole 16-byte vectors).

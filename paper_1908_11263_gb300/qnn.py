@@ -26,7 +26,7 @@ ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
             "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
-            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary")
+            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary", "qconv_hwc_pool2")
 
 
 class QnnError(RuntimeError):
@@ -66,6 +66,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_workspace_size.restype = I32
         lib.qconv_hwc.argtypes = [DP, P, P, P, P, P, P, P, P, SZ, P]
         lib.qconv_hwc.restype = I32
+        lib.qconv_hwc_pool2.argtypes = [DP, P, P, P, P, P, P, P, P, SZ, P]
+        lib.qconv_hwc_pool2.restype = I32
         lib.qconv_hwc_prepare.argtypes = [DP, P, P, P, P, P, P, SZ, P]
         lib.qconv_hwc_prepare.restype = I32
         lib.qconv_hwc_run.argtypes = [DP, P, P, P, SZ, P]
@@ -195,6 +197,41 @@ def conv_hwc(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, strid
     st = load().qconv_hwc(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(bias), _ptr(kappa), _ptr(lam), _ptr(shifts),
                           _ptr(out), _ptr(workspace), ctypes.c_size_t(nbytes), _stream(stream))
     _check(st, "qconv_hwc")
+    return out
+
+
+def conv_hwc_pool2(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, pad=0, out=None, workspace=None,
+                   stream=None):
+    """Quantized HWC convolution (stride 1) with fused compression and 2x2 stride-2 max-pooling
+    (qconv_hwc_pool2); returns uint8 [n, oh // 2, ow // 2, m*Q/8]."""
+    _dev(x, torch.uint8, "x")
+    _dev(w, (torch.int8, torch.uint8), "w")
+    _dev(kappa, torch.int16, "kappa")
+    _dev(lam, torch.int32, "lambda")
+    if bias is not None:
+        _dev(bias, torch.int32, "bias")
+    if shifts is not None:
+        _dev(shifts, torch.uint8, "shifts")
+    per = 8 // bits
+    n, h, wd, cb = x.shape
+    m, kh, kw, cb2 = w.shape
+    if cb != cb2:
+        raise ValueError("x and w disagree on the channel count")
+    desc = conv_desc(n, h, wd, cb * per, m, kh, kw, 1, pad, bits, shift, ALGO_AUTO)
+    oh = h + 2 * desc.pad_h - kh + 1
+    ow = wd + 2 * desc.pad_w - kw + 1
+    if out is None:
+        out = torch.empty((n, oh // 2, ow // 2, m // per), dtype=torch.uint8, device=x.device)
+    else:
+        _dev(out, torch.uint8, "out")
+    nbytes = workspace_size(desc)
+    if workspace is None:
+        workspace = _workspace(nbytes, x.device, stream)
+    elif workspace.numel() < nbytes:
+        raise ValueError("workspace too small")
+    st = load().qconv_hwc_pool2(ctypes.byref(desc), _ptr(x), _ptr(w), _ptr(bias), _ptr(kappa), _ptr(lam),
+                                _ptr(shifts), _ptr(out), _ptr(workspace), ctypes.c_size_t(nbytes), _stream(stream))
+    _check(st, "qconv_hwc_pool2")
     return out
 
 

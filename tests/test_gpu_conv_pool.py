@@ -1,0 +1,134 @@
+"""Fused convolution + 2x2 stride-2 max-pooling (qconv_hwc_pool2) against the oracle's two
+layers in sequence (Sec. IV-A), bit for bit, plus its argument checks (without a GPU)."""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_1908_11263_gb300 import build as qbuild
+from paper_1908_11263_gb300 import qnn
+from gpu_util import THREADS, check_guard, first_mismatch, guarded_output, pack_gpu, to_dev
+
+FAKE = 0x10000  # 16-byte aligned, never dereferenced: validation fails first
+
+
+def spread_case(seed, n, h, w, c, m, k, bits, per_channel_shift):
+    """Seeded layer whose outputs spread over [0, 2^Q - 1]: the bias cancels the accumulators'
+    mean (weights average -1/2), kappa is positive and the shift matches their spread."""
+    rng = np.random.default_rng(seed)
+    top = (1 << bits) - 1
+    x = rng.integers(0, top + 1, size=(n, h, w, c))
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, k, k, c))
+    taps = k * k * c
+    centre = taps * top // 4
+    spread = int(np.sqrt(taps) * ((top + 1) ** 2 - 1) / 12) + 1
+    bias = (centre + rng.integers(-spread, spread + 1, size=m)).astype(np.int32)
+    kappa = rng.integers(1, 400, size=m).astype(np.int16)
+    shift = max(2, int(np.log2(spread * 400 / (top + 1))) + 1)
+    lam = rng.integers(0, (top + 1) << (shift - 1), size=m).astype(np.int32)
+    shifts = rng.integers(shift - 2, shift + 3, size=m).astype(np.uint8) if per_channel_shift else None
+    return x, wt, bias, kappa, lam, shifts, shift
+
+
+def packed_dev(v, bits, shape):
+    per = 8 // bits
+    t = pack_gpu(v.reshape(-1), bits)
+    return t.view(*shape[:-1], shape[-1] // per)
+
+
+def run_fused(x, wt, bias, kappa, lam, shifts, shift, bits, pad):
+    n, h, w, c = x.shape
+    m, k, _, _ = wt.shape
+    per = 8 // bits
+    oh, ow = h + 2 * pad - k + 1, w + 2 * pad - k + 1
+    out, buf = guarded_output((n, oh // 2, ow // 2, m // per))
+    wd = packed_dev(wt, bits, wt.shape)
+    if bits == 8:
+        wd = wd.view(torch.int8)
+    qnn.conv_hwc_pool2(packed_dev(x, bits, x.shape), wd, to_dev(kappa, torch.int16), to_dev(lam, torch.int32),
+                       bias=to_dev(bias, torch.int32), shifts=None if shifts is None else to_dev(shifts, torch.uint8),
+                       shift=shift, bits=bits, pad=pad, out=out)
+    qnn.device_status()
+    check_guard(buf)
+    return out, wd
+
+
+def run_oracle(x, wt, bias, kappa, lam, shifts, shift, bits, pad):
+    n, h, w, c = x.shape
+    m, k, _, _ = wt.shape
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=k, kw=k, sh=1, sw=1, ph=pad, pw=pad, bits=bits)
+    return oracle.conv_hwc_pool2(oracle.pack(x.reshape(-1), bits), oracle.pack(wt.reshape(-1), bits), shape, bias,
+                                 kappa, lam, shifts=shifts, shift=shift, nthreads=THREADS)
+
+
+# (n, h, w, c, m, k, pad, bits): the CIFAR layers' shapes at small batch, partial strips at the
+# right and bottom, odd output sizes (floor), 1x1 and 5x5 windows, C not a multiple of 8, two
+# output-channel tiles, several channel slabs, sub-byte outputs
+SHAPES = [
+    (2, 32, 32, 3, 32, 5, 2, 8),
+    (2, 16, 16, 32, 32, 5, 2, 8),
+    (3, 8, 8, 32, 64, 5, 2, 8),
+    (2, 16, 16, 32, 64, 3, 1, 8),
+    (1, 30, 20, 32, 48, 5, 2, 8),
+    (2, 15, 13, 16, 24, 3, 1, 8),
+    (1, 12, 12, 32, 136, 3, 1, 8),
+    (1, 10, 10, 128, 64, 3, 1, 8),
+    (2, 9, 11, 16, 16, 1, 0, 8),
+    (2, 16, 16, 32, 64, 3, 1, 4),
+    (1, 13, 18, 64, 32, 3, 1, 4),
+    (2, 9, 9, 64, 64, 3, 0, 2),
+    (1, 14, 22, 32, 32, 3, 1, 2),
+]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: "x".join(map(str, s[:6])) + f"_p{s[6]}_q{s[7]}")
+def test_conv_pool2_matches_oracle(shape):
+    n, h, w, c, m, k, pad, bits = shape
+    case = spread_case(hash(shape) & 0xFFFF, n, h, w, c, m, k, bits, per_channel_shift=(h % 2 == 0))
+    want = run_oracle(*case, bits, pad)
+    out, _ = run_fused(*case, bits, pad)
+    got = out.cpu().numpy().reshape(-1)
+    assert first_mismatch(got, want) is None, first_mismatch(got, want)
+    assert len(np.unique(want)) > 4, "pooled outputs nearly constant: the check is weak"
+
+
+@pytest.mark.gpu
+def test_conv_pool2_equals_conv_then_qmaxpool_on_gpu():
+    """The fused kernel against the library's own two launches (qconv_hwc, then qmaxpool)."""
+    n, h, w, c, m, k, pad, bits = 4, 32, 32, 32, 64, 5, 2, 8
+    x, wt, bias, kappa, lam, shifts, shift = spread_case(99, n, h, w, c, m, k, bits, True)
+    fused, wd = run_fused(x, wt, bias, kappa, lam, shifts, shift, bits, pad)
+    full = qnn.conv_hwc(packed_dev(x, bits, x.shape), wd, to_dev(kappa, torch.int16), to_dev(lam, torch.int32),
+                        bias=to_dev(bias, torch.int32), shifts=to_dev(shifts, torch.uint8), shift=shift, bits=bits,
+                        pad=pad)
+    two_step = qnn.maxpool(full, 2, 2, bits=bits)
+    torch.cuda.synchronize()
+    assert torch.equal(fused, two_step)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    qbuild.build()
+    return qnn.load()
+
+
+def test_conv_pool2_rejects_what_it_cannot_run(lib):
+    """Argument checks only (no CUDA call is reached), so this runs without a GPU."""
+    P = ctypes.c_void_p
+
+    def status(d, x=FAKE, y=FAKE, ws=FAKE):
+        return lib.qconv_hwc_pool2(ctypes.byref(d), P(x), P(FAKE), P(FAKE), P(FAKE), P(FAKE), None, P(y), P(ws),
+                                   ctypes.c_size_t(1 << 30), None)
+
+    ok = qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 1, 1, 8, 10)
+    # stride 2 has no tensor-core kernel; a forced CUDA-core kernel has no fused pool
+    assert status(qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 2, 1, 8, 10)) == qnn.QNN_EUNSUPPORTED
+    assert status(qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 1, 1, 8, 10, qnn.ALGO_DIRECT)) == qnn.QNN_EUNSUPPORTED
+    # a 1-pixel-wide output has no pooled pixel
+    assert status(qnn.conv_desc(1, 8, 3, 32, 32, 3, 3, 1, 0, 8, 10)) == qnn.QNN_EINVAL
+    assert status(ok, x=0) == qnn.QNN_EINVAL
+    assert status(ok, y=FAKE + 8) == qnn.QNN_EALIGN
+    assert status(ok, ws=0) == qnn.QNN_EWORKSPACE

@@ -216,6 +216,35 @@ def test_full_layer_against_independent_reference(bits):
         np.testing.assert_array_equal(yp[r], want[b, oy, ox])
 
 
+@pytest.mark.parametrize("bits", [8, 4, 2])
+def test_conv_pool2_against_independent_reference(bits):
+    """A conv layer and then a 2x2 stride-2 max-pool over its quantized output (Sec. IV-A): the
+    independent scatter-form layer above, then the maximum of every window written as four
+    explicit comparisons.  Odd output sizes check the floor rule (the last row and column drop)."""
+    n, h, w, c, m, k = 2, 7, 5, 8, 8, 3
+    x, wt = rand_layer(n, h, w, c, m, k, bits)
+    bias = rng.integers(-50, 50, m)
+    kappa = rng.integers(-5, 40, m)
+    lam = rng.integers(-300, 300, m)
+    shifts = rng.integers(0, 8, m)
+    t = full_layer_ref(x, wt, bias, kappa, lam, shifts, bits, (1, 1), (1, 1))  # [n, 7, 5, m]
+    assert len(np.unique(t)) > 2, "layer outputs nearly constant: the pooling check would be weak"
+    want = np.empty((n, 3, 2, m), np.int64)
+    for b, py, px, o in np.ndindex(want.shape):
+        a0, a1 = t[b, 2 * py, 2 * px, o], t[b, 2 * py, 2 * px + 1, o]
+        a2, a3 = t[b, 2 * py + 1, 2 * px, o], t[b, 2 * py + 1, 2 * px + 1, o]
+        best = a0
+        for v in (a1, a2, a3):
+            if v > best:
+                best = v
+        want[b, py, px, o] = best
+    shape = dict(n=n, h=h, w=w, c=c, m=m, kh=k, kw=k, sh=1, sw=1, ph=1, pw=1, bits=bits)
+    y = oracle.conv_hwc_pool2(oracle.pack(x.reshape(-1), bits), oracle.pack(wt.reshape(-1), bits), shape, bias,
+                              kappa, lam, shifts=shifts)
+    got = oracle.unpack(y, want.size, bits, False).reshape(want.shape)
+    np.testing.assert_array_equal(got, want)
+
+
 def test_zero_weights_give_bias_only_output():
     n, h, w, c, m = 1, 4, 4, 8, 4
     x, _ = rand_layer(n, h, w, c, m, 3)
