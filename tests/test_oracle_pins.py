@@ -222,13 +222,19 @@ def test_conv_pool2_against_independent_reference(bits):
     independent scatter-form layer above, then the maximum of every window written as four
     explicit comparisons.  Odd output sizes check the floor rule (the last row and column drop)."""
     n, h, w, c, m, k = 2, 7, 5, 8, 8, 3
-    x, wt = rand_layer(n, h, w, c, m, k, bits)
-    bias = rng.integers(-50, 50, m)
-    kappa = rng.integers(-5, 40, m)
-    lam = rng.integers(-300, 300, m)
-    shifts = rng.integers(0, 8, m)
+    g = np.random.default_rng(1000 + bits)  # own stream: the case does not depend on test order
+    top = (1 << bits) - 1
+    x = g.integers(0, top + 1, size=(n, h, w, c))
+    wt = g.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, k, k, c))
+    # centre the accumulators (weights average -1/2) and scale their spread onto [0, top]
+    shift = {8: 13, 4: 8, 2: 5}[bits]
+    bias = k * k * c * top // 4 + g.integers(-20, 21, m)
+    kappa = g.integers(10, 30, m)
+    lam = (top // 2) << shift
+    lam = lam + g.integers(-(1 << (shift - 1)), 1 << (shift - 1), m)
+    shifts = np.full(m, shift)
     t = full_layer_ref(x, wt, bias, kappa, lam, shifts, bits, (1, 1), (1, 1))  # [n, 7, 5, m]
-    assert len(np.unique(t)) > 2, "layer outputs nearly constant: the pooling check would be weak"
+    assert len(np.unique(t)) > min(top, 6), "layer outputs nearly constant: the pooling check would be weak"
     want = np.empty((n, 3, 2, m), np.int64)
     for b, py, px, o in np.ndindex(want.shape):
         a0, a1 = t[b, 2 * py, 2 * px, o], t[b, 2 * py, 2 * px + 1, o]
