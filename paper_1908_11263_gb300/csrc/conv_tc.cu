@@ -139,6 +139,8 @@ struct TcArgs {
     FastDiv fd_ncb;
     int conv_fast;                            // converter fast path (see ConvItem)
     int pool, pool_oh, pool_ow;               // fused 2x2/2 max-pool and its output height, width
+    int fp8;                                  // e4m3 staging and kind::f8f6f4 MMAs (INT-4/INT-2)
+    int kch;                                  // channels per 16-byte K-chunk: 8 (fp16) or 16 (e4m3)
     int mma_warps;                            // 2: warps 12 and 15 issue alternate tiles
     const int32_t *thr;                       // staircase thresholds in the workspace, or null
     uint32_t off_thr;                         // their shared-memory copy
@@ -489,7 +491,7 @@ __device__ __forceinline__ ConvItem conv_item(const TcArgs &a, const ConvMap &mp
     const int ncol = a.ncol_w << a.log2_groups;
     const int ci = mp.ci0;
     const int gq = ci / a.ncol_w;  // once per kernel
-    const int c0 = gq * 8;
+    const int c0 = gq * a.kch;
     it.px = ci - gq * a.ncol_w;
     it.c0 = c0;
     it.active = ci < ncol;
@@ -507,6 +509,35 @@ __device__ __forceinline__ ConvItem conv_item(const TcArgs &a, const ConvMap &mp
     return it;
 }
 
+// e4m3 codes of four 4-bit values v0..v3 (selector nibbles, bits 0-15): value
+// v goes to byte k.  Two 8-entry lookups: prmt picks byte v & 7 of a table,
+// and a selector nibble with bit 3 set yields that byte's sign, 0 here, so
+// each lookup answers for its own half of 0..15 and zero for the other.  The
+// tables hold e4m3(v) = 2^(E-7) * (1 + M/8) for v = 0..7 and 8..15, all exact.
+__device__ __forceinline__ uint32_t e4m3x4(uint32_t sel)
+{
+    return prmt(0x44403800u, 0x4E4C4A48u, sel) | prmt(0x53525150u, 0x57565554u, sel ^ 0x8888u);
+}
+
+// 16 unsigned INT-4 (one 8-byte load) or INT-2 (one 4-byte load) activations
+// -> 16 e4m3 bytes.  INT-4 keeps the channel order; INT-2 yields channels
+// {0,2,4,6}, {1,3,5,7}, {8,10,12,14}, {9,11,13,15} in its four words (the
+// filters are laid out to match).
+template <int BITS>
+__device__ __forceinline__ uint4 cvt_raw_f8(const uint8_t *p)
+{
+    uint4 r;
+    if (BITS == 4) {
+        const uint2 v = *reinterpret_cast<const uint2 *>(p);
+        r = make_uint4(e4m3x4(v.x), e4m3x4(v.x >> 16), e4m3x4(v.y), e4m3x4(v.y >> 16));
+    } else {
+        const uint32_t v = *reinterpret_cast<const uint32_t *>(p);
+        const uint32_t ev = v & 0x33333333u, od = (v >> 2) & 0x33333333u;  // crumbs 2k and 2k+1 as nibbles
+        r = make_uint4(e4m3x4(ev), e4m3x4(od), e4m3x4(ev >> 16), e4m3x4(od >> 16));
+    }
+    return r;
+}
+
 template <int BITS>
 __device__ __forceinline__ uint4 cvt_raw(const uint8_t *p)
 {
@@ -519,13 +550,13 @@ __device__ __forceinline__ uint4 cvt_raw(const uint8_t *p)
 // per pass with every load issued before the stores.  The values written are
 // those of convert_stage(): the staged encoding inside the image, the encoded
 // zero outside it; row tiles store the copies in jmask, strips one position.
-template <int BITS, int NJ, bool STRIP>
+template <int BITS, int NJ, bool STRIP, bool F8>
 __device__ __forceinline__ void convert_fast(const TcArgs &a, const uint8_t *raw, uint8_t *stage, const TileGeo &g,
                                              const ConvItem &it, const ConvMap &mp, int slab)
 {
     // a group wholly past C keeps the encoded zero written at kernel start
     if (!it.active || slab * a.cs + it.c0 >= a.c) return;
-    const uint32_t padv = pad_half2<BITS>();
+    const uint32_t padv = F8 ? 0u : pad_half2<BITS>();
     const int nph = mp.nphase;
     const int row_bytes = static_cast<int>(a.row_bytes);
     bool col_ok = true;
@@ -551,7 +582,8 @@ __device__ __forceinline__ void convert_fast(const TcArgs &a, const uint8_t *raw
         for (int u = 0; u < kRowsPerPass; ++u) {
             const int rr = r + u * nph;
             const bool ok = col_ok && rr >= g.r_lo && rr < g.r_hi;
-            const uint4 x = cvt_raw<BITS>(ok ? src + u * src_step : raw);
+            const uint8_t *q = ok ? src + u * src_step : raw;
+            const uint4 x = F8 ? cvt_raw_f8<BITS>(q) : cvt_raw<BITS>(q);
             v[u] = ok ? x : make_uint4(padv, padv, padv, padv);
         }
 #pragma unroll
@@ -576,7 +608,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
     const ConvMap mp = conv_map(a.ncol_w << a.log2_groups);
     // encoded zero everywhere once: padding columns are never written afterwards
     {
-        const uint32_t padv = pad_half2<BITS>();
+        const uint32_t padv = a.fp8 ? 0u : pad_half2<BITS>();  // e4m3 zero is 0
         const uint4 pad4 = make_uint4(padv, padv, padv, padv);
         const uint32_t total = a.stages * a.stage_bytes / 16;
         for (uint32_t i = threadIdx.x; i < total; i += 128) sts128(stages_base + i * 16, pad4);
@@ -598,14 +630,27 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
         for (int slab = 0; slab < a.nslab; ++slab) {
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
             uint8_t *st = smem + a.off_stages + stage * a.stage_bytes;
-            if (!a.conv_fast)
+            bool staged = false;
+            if constexpr (BITS != 8) {
+                if (a.fp8) {  // always on the fast path (planner)
+                    if (a.strip)
+                        convert_fast<BITS, 1, true, true>(a, raw, st, g, item, mp, slab);
+                    else if (a.kw <= 3)
+                        convert_fast<BITS, 3, false, true>(a, raw, st, g, item, mp, slab);
+                    else
+                        convert_fast<BITS, 5, false, true>(a, raw, st, g, item, mp, slab);
+                    staged = true;
+                }
+            }
+            if (staged) {
+            } else if (!a.conv_fast)
                 convert_stage<BITS>(a, raw, st, g, slab, vec, mp);
             else if (a.strip)
-                convert_fast<BITS, 1, true>(a, raw, st, g, item, mp, slab);
+                convert_fast<BITS, 1, true, false>(a, raw, st, g, item, mp, slab);
             else if (a.kw <= 3)
-                convert_fast<BITS, 3, false>(a, raw, st, g, item, mp, slab);
+                convert_fast<BITS, 3, false, false>(a, raw, st, g, item, mp, slab);
             else
-                convert_fast<BITS, 5, false>(a, raw, st, g, item, mp, slab);
+                convert_fast<BITS, 5, false, false>(a, raw, st, g, item, mp, slab);
             if (threadIdx.x == 0) stage_info[stage] = info;  // released by this thread's arrive below
             fence_proxy_async_smem();
             mbar_arrive(&a_full[stage]);
@@ -708,7 +753,7 @@ __device__ __forceinline__ void b_loader_role(const TcArgs &a, uint8_t *smem, ui
                     ok = false;
                     break;
                 }
-                const int kchunk = (tap * a.c_pad + slab * a.cs) / 8;
+                const int kchunk = (tap * a.c_pad + slab * a.cs) / a.kch;
                 bulk_copy(smem + bs * a.b_tile_bytes, wsrc + static_cast<size_t>(kchunk) * nt_cols * 16,
                           a.b_tile_bytes, &b_full[bs]);
                 ++issued;
@@ -730,7 +775,7 @@ __device__ __forceinline__ void b_loader_role(const TcArgs &a, uint8_t *smem, ui
 // Descriptors come from uniform values only (tap offsets live in the kernel's
 // parameter block), and the loop body has no conditionals, so the MMAs go out
 // back to back.
-template <int KSTEPS>
+template <int KSTEPS, bool F8>
 __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t a_tmpl, uint64_t b_tmpl,
                                            uint32_t abase, uint32_t bbase, uint32_t tap_b16, uint32_t a_step,
                                            uint32_t b_step, int t0, int t1, uint32_t idesc)
@@ -740,7 +785,10 @@ __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t
         const uint64_t ad = a_tmpl + (abase + a.tap_a16[t]);
         const uint64_t bd = b_tmpl + (bbase + t * tap_b16);
 #pragma unroll
-        for (int kk = 0; kk < KSTEPS; ++kk) mma_f16_ss_warp(d, ad + kk * a_step, bd + kk * b_step, idesc, 1u);
+        for (int kk = 0; kk < KSTEPS; ++kk) {
+            if (F8) mma_f8_ss_warp(d, ad + kk * a_step, bd + kk * b_step, idesc, 1u);
+            else mma_f16_ss_warp(d, ad + kk * a_step, bd + kk * b_step, idesc, 1u);
+        }
     }
 }
 
@@ -754,7 +802,7 @@ __device__ __forceinline__ void issue_taps(const TcArgs &a, uint32_t d, uint64_t
 // the CTA's tiles sel, sel + 2, ...; stage, group and their phases follow from
 // the tile's position in the CTA's sequence, so one issuer's waits and commits
 // overlap the other's MMAs.
-template <int KSTEPS>
+template <int KSTEPS, bool F8>
 __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem, uint32_t tmem_base,
                                                   uint64_t *a_full, uint64_t *a_empty, uint64_t *b_full,
                                                   uint64_t *b_empty, uint64_t *acc_full, uint64_t *acc_empty,
@@ -767,7 +815,7 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
     const uint32_t b16 = smem_addr(smem) >> 4;
     const uint32_t stage16 = a.stage_bytes >> 4;
     const uint32_t a_step = 2 * (a.chunk_stride >> 4), b_step = 2 * nt_cols;
-    const uint32_t tap_b16 = (a.c_pad / 8) * nt_cols;
+    const uint32_t tap_b16 = (a.c_pad / a.kch) * nt_cols;
     const int chunk_taps = a.chunk_mmas / KSTEPS, taps = a.kh * a.kw;
     const int ngroups = a.ngroups, grp_chunks = a.grp_chunks, nsg = a.nsg, nchunks = a.nchunks;
     const int nstages = a.stages;
@@ -805,7 +853,7 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
             const int last_chunk = min(nchunks, (sg + 1) * grp_chunks);
             for (int c = sg * grp_chunks; c < last_chunk; ++c) {
                 const int t1 = min(t0 + chunk_taps, taps);
-                issue_taps<KSTEPS>(a, d, a_tmpl, b_tmpl, abase, b16, tap_b16, a_step, b_step, t0, t1, idesc);
+                issue_taps<KSTEPS, F8>(a, d, a_tmpl, b_tmpl, abase, b16, tap_b16, a_step, b_step, t0, t1, idesc);
                 t0 = t1;
                 d += nt_cols;
             }
@@ -821,6 +869,7 @@ __device__ __forceinline__ void mma_role_resident(const TcArgs &a, uint8_t *smem
 }
 
 // MMA issue, general case (streamed filters, or several channel slabs per tile).
+template <bool F8>
 __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *a_full,
                                          uint64_t *a_empty, uint64_t *b_full, uint64_t *b_empty, uint64_t *acc_full,
                                          uint64_t *acc_empty, uint64_t *done, const volatile uint32_t *stage_info,
@@ -832,12 +881,12 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
     const uint32_t stages16 = smem_addr(smem + a.off_stages) >> 4;
     const uint32_t b16 = smem_addr(smem) >> 4;
     const uint32_t stage16 = a.stage_bytes >> 4, btile16 = a.b_tile_bytes >> 4;
-    const uint32_t a_step = 2 * (a.chunk_stride >> 4), b_step = 2 * nt_cols;  // one k-step = two 8-channel chunks
-    const uint32_t slab_b16 = (a.cs / 8) * nt_cols;
-    const int ksteps = a.cs / 16;
+    const uint32_t a_step = 2 * (a.chunk_stride >> 4), b_step = 2 * nt_cols;  // one k-step = two K-chunks
+    const uint32_t slab_b16 = (a.cs / a.kch) * nt_cols;
+    const int ksteps = a.cs / (2 * a.kch);
     const bool resident = a.b_resident != 0;
-    // resident filters: tap t of slab s sits at t * c_pad/8 chunks; streamed: each tap has its own tile
-    const uint32_t tap_b16 = resident ? (a.c_pad / 8) * nt_cols : 0;
+    // resident filters: tap t of slab s sits at t * c_pad/kch chunks; streamed: each tap has its own tile
+    const uint32_t tap_b16 = resident ? (a.c_pad / a.kch) * nt_cols : 0;
     const int chunk_taps = a.chunk_mmas / ksteps, taps = a.kh * a.kw;
     const int nslab = a.nslab, nstages = a.stages, nbstages = a.b_stages;
     const int grp_chunks = a.grp_chunks, ngroups = a.ngroups, nchunks = a.nchunks;
@@ -889,11 +938,11 @@ __device__ __forceinline__ void mma_role(const TcArgs &a, uint8_t *smem, uint32_
                 seg = min(seg, chunk_taps - in_chunk);
                 const uint32_t d = tmem_base + (grp * grp_chunks + sub) * nt_cols;
                 if (ksteps == 1)
-                    issue_taps<1>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                    issue_taps<1, F8>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
                 else if (ksteps == 2)
-                    issue_taps<2>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                    issue_taps<2, F8>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
                 else
-                    issue_taps<4>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
+                    issue_taps<4, F8>(a, d, a_tmpl, b_tmpl, abase, bbase, tap_b16, a_step, b_step, tap, tap + seg, idesc);
                 tap += seg;
                 in_chunk += seg;
                 if (in_chunk == chunk_taps || (slab == nslab - 1 && tap == taps)) {  // chunk complete
@@ -1342,20 +1391,38 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     } else if (warp < kConvWarps + kEpiWarps) {
         epilogue_role<BITS, NT, POOL>(a, smem, tmem_base, acc_full, acc_empty);
     } else if (warp == kMmaWarp || (warp == kMmaWarp2 && a.mma_warps == 2)) {
+        // the instruction descriptor is the same for both kinds (format fields 0: f16 / e4m3)
         const uint32_t idesc = idesc_f16_f32(kTileM, NT);
         const int sel = warp == kMmaWarp ? 0 : 1;
-        if (a.b_resident && a.nslab == 1 && a.cs == 32)
-            mma_role_resident<2>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                 stage_info, idesc, NT, sel, a.mma_warps);
-        else if (a.b_resident && a.nslab == 1 && a.cs == 64)
-            mma_role_resident<4>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                 stage_info, idesc, NT, sel, a.mma_warps);
+        const int ks = a.cs / (2 * a.kch);  // k-steps per tap and slab
+        bool issued = false;
+        if constexpr (BITS != 8) {
+            if (a.fp8) {
+                if (a.b_resident && a.nslab == 1 && ks == 1)
+                    mma_role_resident<1, true>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full,
+                                               acc_empty, done, stage_info, idesc, NT, sel, a.mma_warps);
+                else if (a.b_resident && a.nslab == 1 && ks == 2)
+                    mma_role_resident<2, true>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full,
+                                               acc_empty, done, stage_info, idesc, NT, sel, a.mma_warps);
+                else
+                    mma_role<true>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                   stage_info, idesc, NT);
+                issued = true;
+            }
+        }
+        if (issued) {
+        } else if (a.b_resident && a.nslab == 1 && ks == 2)
+            mma_role_resident<2, false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                        stage_info, idesc, NT, sel, a.mma_warps);
+        else if (a.b_resident && a.nslab == 1 && ks == 4)
+            mma_role_resident<4, false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                        stage_info, idesc, NT, sel, a.mma_warps);
         else if (a.b_resident && a.nslab == 1)
-            mma_role_resident<1>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                 stage_info, idesc, NT, sel, a.mma_warps);
+            mma_role_resident<1, false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                        stage_info, idesc, NT, sel, a.mma_warps);
         else
-            mma_role(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info, idesc,
-                     NT);
+            mma_role<false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info,
+                            idesc, NT);
     } else if (warp == kRawWarp) {
         raw_loader_role(a, smem, raw_full, raw_empty);
     } else if (warp == kBWarp) {
@@ -1417,11 +1484,23 @@ __device__ bool saturation_bounds(long long kappa, long long lambda, int s, long
 // [0, 2^Q-1]); mode "clamp" when the saturation bounds allow a 32-bit form.
 // The kernel lets the convolution that follows it start at once (that kernel
 // waits for these results only where it reads them).
+// e4m3 code of an integer with |v| <= 15 (exact): sign, exponent e + 7 for
+// |v| in [2^e, 2^(e+1)), three fraction bits.
+__device__ __forceinline__ uint8_t e4m3_of_int(int v)
+{
+    if (v == 0) return 0;
+    const uint32_t sgn = v < 0 ? 0x80u : 0u;
+    const uint32_t mag = static_cast<uint32_t>(v < 0 ? -v : v);
+    const int e = 31 - __clz(static_cast<int>(mag));
+    const uint32_t frac = ((mag << 3) >> e) & 7u;
+    return static_cast<uint8_t>(sgn | (static_cast<uint32_t>(e + 7) << 3) | frac);
+}
+
 template <int BITS>
 __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, const int32_t *bias, const int16_t *kappa,
                                                            const int32_t *lambda, const uint8_t *shifts, int shift,
                                                            int m, int mp, int kh, int kw, int c, int c_pad, int k_pad,
-                                                           int nt, int nchunks, uint16_t *wpack, int4 *chan,
+                                                           int nt, int nchunks, int fp8, uint16_t *wpack, int4 *chan,
                                                            const int32_t *thresholds, int32_t *thr_out)
 {
     pdl_trigger();
@@ -1449,9 +1528,17 @@ __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, con
             pos += max(v, 0);
             neg += min(v, 0);
             const int k = tap * c_pad + cc;
-            const int slot = BITS == 8 ? (cc & 7) : slot_of[cc & 7];
-            const size_t dst = ((static_cast<size_t>(tile) * (k_pad / 8) + k / 8) * nt + col) * 8 + slot;
-            wpack[dst] = __half_as_ushort(__int2half_rn(v));
+            if (fp8) {
+                // e4m3 bytes, 16 channels per K-chunk; INT-2 in the converter's word order
+                const int ch = cc & 15;
+                const int slot = BITS == 4 ? ch : (ch & 8) + (ch & 1) * 4 + ((ch & 7) >> 1);
+                const size_t dst = ((static_cast<size_t>(tile) * (k_pad / 16) + k / 16) * nt + col) * 16 + slot;
+                reinterpret_cast<uint8_t *>(wpack)[dst] = e4m3_of_int(v);
+            } else {
+                const int slot = BITS == 8 ? (cc & 7) : slot_of[cc & 7];
+                const size_t dst = ((static_cast<size_t>(tile) * (k_pad / 8) + k / 8) * nt + col) * 8 + slot;
+                wpack[dst] = __half_as_ushort(__int2half_rn(v));
+            }
         }
     }
 #pragma unroll
@@ -1467,14 +1554,14 @@ __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, con
     }
     if (lane == 0 && thresholds) {
         // the epilogue compares acc = s + beta (bias is part of the thresholds)
-        const long long off = (BITS == 8) ? -128 : 1024;
+        const long long off = fp8 ? 0 : (BITS == 8) ? -128 : 1024;
         const uint32_t beta = 0u - static_cast<uint32_t>(off * sum) - static_cast<uint32_t>(nchunks) * kMagic;
         chan[o] = make_int4(0, 0, 0, kModeThreshold);  // .x: threshold location, set when staged
         chan[mp + o] = make_int4(static_cast<int32_t>(beta), 0, 0, 0);
     } else if (lane == 0) {
         int4 r0 = make_int4(0, 0, 0, kModeDirect), r1 = make_int4(0, 0, 0, 0);
         if (o < m) {
-            const long long off = (BITS == 8) ? -128 : 1024;  // staged activation = x + off
+            const long long off = fp8 ? 0 : (BITS == 8) ? -128 : 1024;  // staged activation = x + off
             const int32_t b = bias ? bias[o] : 0;
             const uint32_t beta = static_cast<uint32_t>(b) - static_cast<uint32_t>(off * sum) -
                                   static_cast<uint32_t>(nchunks) * kMagic;
@@ -1558,10 +1645,20 @@ size_t chan_offset(const TcPlan &plan)
 
 }  // namespace
 
-TcPlan plan_conv_tc(const ConvShape &s)
+namespace {
+
+// One layout: fp16 staging (K = 16 channels per MMA), or for INT-4/INT-2 with
+// C a multiple of 32, e4m3 staging (K = 32).  The e4m3 embedding is exact: the
+// values lie in [-8, 15], each e4m3 product is an integer up to 15 * 8, and a
+// probe of the kind::f8f6f4 MMA against int64 sums (K up to 1024, adversarial
+// orderings, with and without the accumulator pre-load) found no error.
+TcPlan plan_layout(const ConvShape &s, bool fp8)
 {
     TcPlan p{};
     p.ok = false;
+    p.fp8 = fp8;
+    const int kch = fp8 ? 16 : 8;  // channels per 16-byte K-chunk
+    const uint32_t eb = fp8 ? 1 : 2;  // bytes per staged element
     if (s.sh != 1 || s.sw != 1 || s.oh <= 0 || s.ow <= 0) return p;
     if (s.kh * s.kw > kMaxTaps || s.kw > 32) return p;  // per-tap table; 32-bit copy mask
     const long long row_bytes = static_cast<long long>(s.w) * s.c * s.bits / 8;
@@ -1569,7 +1666,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
     const int mp16 = (s.m + 15) / 16 * 16;
     p.nt = mp16 <= 16 ? 16 : mp16 <= 32 ? 32 : mp16 <= 64 ? 64 : 128;
     p.n_ntiles = (s.m + p.nt - 1) / p.nt;
-    p.c_pad = (s.c + 15) / 16 * 16;
+    p.c_pad = (s.c + 2 * kch - 1) / (2 * kch) * (2 * kch);
     p.k_pad = s.kh * s.kw * p.c_pad;
     p.row_bytes = static_cast<uint32_t>(row_bytes);
     // A tile's 128 MMA rows are 16 groups of 8 consecutive output pixels of one
@@ -1611,11 +1708,13 @@ TcPlan plan_conv_tc(const ConvShape &s)
     if (p.p_alloc * 16 >= (1 << 18)) return p;  // descriptor offset field
     p.raw_bytes = round_up(static_cast<uint32_t>(p.rows_max * row_bytes), 128);
     if (p.raw_bytes >= (1u << 20)) return p;    // single transaction count
-    p.b_bytes = static_cast<uint32_t>(p.nt) * p.k_pad * 2;
-    p.mmas_per_tile = p.k_pad / 16;
-    // products per exact chunk: |staged x| * |w| <= 2^14 (INT-8), 1039*8 (INT-4), 1027*2 (INT-2)
-    const long long max_prod = s.bits == 8 ? 16384 : s.bits == 4 ? 1039 * 8 : 1027 * 2;
-    const int limit = static_cast<int>(((1ll << 22) / max_prod) / 16);  // MMAs per exact chunk
+    p.b_bytes = static_cast<uint32_t>(p.nt) * p.k_pad * eb;
+    p.mmas_per_tile = p.k_pad / (2 * kch);
+    // products per exact chunk: |staged x| * |w| <= 2^14 (INT-8), 1039*8 (INT-4), 1027*2 (INT-2);
+    // e4m3 staging has no offset: 15*8 (INT-4), 3*2 (INT-2)
+    const long long max_prod = fp8 ? (s.bits == 4 ? 15 * 8 : 3 * 2)
+                                   : s.bits == 8 ? 16384 : s.bits == 4 ? 1039 * 8 : 1027 * 2;
+    const int limit = static_cast<int>(((1ll << 22) / max_prod) / (2 * kch));  // MMAs per exact chunk
     p.limit_mmas = limit;
     const int mp = p.n_ntiles * p.nt;
     const uint32_t thr_bytes = s.thr ? static_cast<uint32_t>(mp) * 4 * kThrStride : 0;
@@ -1624,14 +1723,14 @@ TcPlan plan_conv_tc(const ConvShape &s)
     for (int resident = 1; resident >= 0 && !p.cs; --resident) {
         if (resident && p.b_bytes > 120u * 1024u) continue;
         for (int cs : {64, 32, 16}) {
-            if (cs > p.c_pad || p.c_pad % cs) continue;
+            if (cs > p.c_pad || p.c_pad % cs || cs < 2 * kch) continue;
             for (int stages : {3, 2}) {
                 for (int bst : {4, 3, 2}) {
                     if (resident && bst != 4) continue;
                     const int b_stages = resident ? 1 : bst;
-                    const uint32_t b_tile = static_cast<uint32_t>(p.nt) * cs * 2;
+                    const uint32_t b_tile = static_cast<uint32_t>(p.nt) * cs * eb;
                     const uint32_t b_region = resident ? round_up(p.b_bytes, 128) : b_stages * b_tile;
-                    const uint32_t copy_bytes = static_cast<uint32_t>(p.p_alloc) * cs * 2;
+                    const uint32_t copy_bytes = static_cast<uint32_t>(p.p_alloc) * cs * eb;
                     const uint32_t stage_bytes = copy_bytes * (p.strip ? 1 : s.kw);
                     const uint32_t off_raw = round_up(b_region, 128);
                     const uint32_t off_stages = off_raw + p.raw_stages * p.raw_bytes;
@@ -1666,7 +1765,7 @@ TcPlan plan_conv_tc(const ConvShape &s)
     if (!p.cs) return p;
     {
         // chunks hold whole taps (every k-step of a tap goes to one accumulator)
-        const int ksteps = p.cs / 16, units = p.mmas_per_tile / ksteps;
+        const int ksteps = p.cs / (2 * kch), units = p.mmas_per_tile / ksteps;
         const int limit_units = std::max(1, p.limit_mmas / ksteps);
         int nch = (units + limit_units - 1) / limit_units;
         const int per = (units + nch - 1) / nch;
@@ -1697,6 +1796,20 @@ TcPlan plan_conv_tc(const ConvShape &s)
     return p;
 }
 
+}  // namespace
+
+TcPlan plan_conv_tc(const ConvShape &s)
+{
+    if (s.bits != 8 && s.c % 32 == 0) {
+        // e4m3 staging runs on the converter's fast path only: at most one
+        // 16-channel item per thread and slab, strips or kernels at most 5 wide
+        const TcPlan p = plan_layout(s, true);
+        const int ncol_w = p.strip ? p.sp : s.w;
+        if (p.ok && ncol_w * (p.cs / 16) <= 128 && (p.strip || s.kw <= 5)) return p;
+    }
+    return plan_layout(s, false);
+}
+
 cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
                                 cudaStream_t st)
 {
@@ -1707,7 +1820,7 @@ cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const Co
 #define QNN_PREP(B)                                                                                              \
     conv_tc_prep_kernel<B><<<(mp + 7) / 8, 256, 0, st>>>(p.w, p.bias, p.kappa, p.lambda, p.shifts, p.shift, s.m, \
                                                          mp, s.kh, s.kw, s.c, plan.c_pad, plan.k_pad, plan.nt,   \
-                                                         plan.nchunks, wpack, chan, p.thresholds, thr)
+                                                         plan.nchunks, plan.fp8, wpack, chan, p.thresholds, thr)
     switch (s.bits) {
         case 8: QNN_PREP(8); break;
         case 4: QNN_PREP(4); break;
@@ -1731,7 +1844,12 @@ cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uin
     a.n = s.n; a.h = s.h; a.w = s.w; a.c = s.c; a.m = s.m; a.kh = s.kh; a.kw = s.kw;
     a.ph = s.ph; a.pw = s.pw; a.oh = s.oh; a.ow = s.ow;
     a.c_pad = plan.c_pad; a.cs = plan.cs; a.nslab = plan.nslab;
-    a.log2_groups = plan.cs == 64 ? 3 : plan.cs == 32 ? 2 : 1;
+    a.fp8 = plan.fp8;
+    a.kch = plan.fp8 ? 16 : 8;
+    {
+        const int groups = plan.cs / a.kch;  // K-chunks per slab
+        a.log2_groups = groups == 8 ? 3 : groups == 4 ? 2 : 1;
+    }
     a.n_ntiles = plan.n_ntiles; a.tiles_per_img = plan.tiles_per_img;
     a.total_tiles = static_cast<int>(plan.total_tiles);
     a.rows_max = plan.rows_max; a.p_alloc = plan.p_alloc;

@@ -164,6 +164,20 @@ __device__ __forceinline__ void mma_f16_ss_warp(uint32_t d_tmem, uint64_t a_desc
         : "memory");
 }
 
+// As mma_f16_ss_warp with kind::f8f6f4: A and B e4m3 (instruction-descriptor
+// format fields 0), K = 32 per MMA, fp32 accumulator.
+__device__ __forceinline__ void mma_f8_ss_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                               uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 __device__ __forceinline__ void mma_commit_warp(uint64_t *bar)
 {
     asm volatile(

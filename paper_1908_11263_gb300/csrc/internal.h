@@ -49,6 +49,7 @@ struct TcPlan {
     int b_resident;     // whole filter set kept in shared memory
     int tiles_per_img;  // row tiles: ceil(oh * ow / 128); strips: ceil(oh / 16) * ceil(ow / 8)
     int strip;          // 16 x 8 strip tiles staged as one padded window (else 128-pixel row tiles)
+    int fp8;            // INT-4/INT-2 staged as e4m3 bytes, kind::f8f6f4 MMAs with K = 32 (else fp16, K = 16)
     int sp;             // strips: window width in pixels (8 + kw - 1)
     int ncb;            // strips: column blocks per image
     long long total_tiles;

@@ -98,6 +98,34 @@ def test_conv_shift_extremes(shift):
         assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
 
 
+@pytest.mark.parametrize("bits", [4, 2])
+@pytest.mark.parametrize("k,c", [(3, 32), (3, 256), (1, 256)])
+@pytest.mark.parametrize("pick", ["max_neg", "max_pos", "mixed"])
+def test_subbyte_exact_accumulation_at_the_bounds(bits, k, c, pick):
+    """Sub-byte layers with C a multiple of 32 stage e4m3 bytes and run kind::f8f6f4 MMAs. Constant
+    activations at the top of the range, with weights at either end of theirs, drive every
+    accumulator to its extreme (K up to 2304). With kappa=1, shift=0 and lambda = 1 - acc, every
+    output reads 1 only if the accumulator is exact."""
+    n, m = 1, 16
+    top, lo, hi = (1 << bits) - 1, -(1 << (bits - 1)), (1 << (bits - 1)) - 1
+    h, w = (4, 32) if k == 1 else (6, 6)
+    x = np.full((n, h, w, c), top)
+    wval = {"max_neg": lo, "max_pos": hi, "mixed": lo}[pick]
+    wt = np.full((m, k, k, c), wval)
+    if pick == "mixed":  # alternate the extremes along K and flip them across channels
+        wt[..., 1::2] = hi
+        wt[1::2] = lo + hi - wt[1::2]
+    acc = (top * wt.reshape(m, -1).sum(axis=1)).astype(np.int64)
+    lam = (1 - acc).astype(np.int32)
+    kappa = np.ones(m, np.int16)
+    assert qnn.conv_algo(qnn.conv_desc(n, h, w, c, m, k, k, 1, 0, bits, 0)) == qnn.ALGO_TENSORCORE
+    got = conv_gpu(x, wt, None, kappa, lam, None, 0, bits, (1, 1), (0, 0), qnn.ALGO_TENSORCORE)
+    want = conv_oracle(x, wt, None, kappa, lam, None, 0, bits, (1, 1), (0, 0))
+    assert first_mismatch(got, want) is None, first_mismatch(got, want)
+    per = 8 // bits
+    assert np.all(oracle.unpack(want, want.size * per, bits, False) == 1)
+
+
 @pytest.mark.parametrize("xval,wval", [(0, -128), (255, 127), (255, -128), (0, 127), (128, -128), (1, -1)])
 @pytest.mark.parametrize("k,c", [(1, 256), (3, 128), (3, 256)])
 def test_exact_accumulation_at_the_bounds(xval, wval, k, c):
