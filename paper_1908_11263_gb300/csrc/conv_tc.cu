@@ -599,7 +599,7 @@ __device__ __forceinline__ void convert_fast(const TcArgs &a, const uint8_t *raw
     }
 }
 
-template <int BITS>
+template <int BITS, bool LEAN>
 __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
                                uint64_t *a_full, uint64_t *a_empty, volatile uint32_t *stage_info)
 {
@@ -643,7 +643,7 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
                 }
             }
             if (staged) {
-            } else if (!a.conv_fast)
+            } else if (!LEAN && !a.conv_fast)  // the lean kernel runs only fast-path plans
                 convert_stage<BITS>(a, raw, st, g, slab, vec, mp);
             else if (a.strip)
                 convert_fast<BITS, 1, true, false>(a, raw, st, g, item, mp, slab);
@@ -1160,7 +1160,7 @@ __device__ __forceinline__ void release_acc(uint64_t *bar)
 // back and releases the group before the compression arithmetic, so the MMA
 // warp can refill it meanwhile.  Tiles that take several groups carry their
 // running sums in TMEM.
-template <int BITS, int NT, bool POOL>
+template <int BITS, int NT, bool POOL, bool LEAN>
 __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
                                               uint64_t *acc_empty)
 {
@@ -1259,24 +1259,24 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
             uint32_t v[CW];
             bool drained = false;
             if constexpr (CW == 32) {
-                if (nsg == 1 && nsub == 2) {
-                    // the whole tile in one group of two buffers: per half of
-                    // the warp's columns, both buffers' loads in flight, one wait
+                if (nsg == 1 && nsub <= 2) {
+                    // the whole tile in one group of one or two buffers: per
+                    // half of the warp's columns, every load in flight, one wait
 #pragma unroll
                     for (int b0 = 0; b0 < 32; b0 += 16) {
                         uint32_t t0[16], t1[16];
                         tmem_ld16(grp_addr + b0, t0);
-                        tmem_ld16(grp_addr + NT + b0, t1);
+                        if (nsub == 2) tmem_ld16(grp_addr + NT + b0, t1);
                         tmem_wait_ld();
 #pragma unroll
-                        for (int k = 0; k < 16; ++k) v[b0 + k] = t0[k] + t1[k];
+                        for (int k = 0; k < 16; ++k) v[b0 + k] = nsub == 2 ? t0[k] + t1[k] : t0[k];
                         tmem_st16_fill(grp_addr + b0, kMagic);
-                        tmem_st16_fill(grp_addr + NT + b0, kMagic);
+                        if (nsub == 2) tmem_st16_fill(grp_addr + NT + b0, kMagic);
                     }
                     drained = true;
                 }
             }
-            if (!drained) {
+            if (!LEAN && !drained) {  // the lean kernel runs only one-group, at most two-buffer plans
 #pragma unroll
             for (int k = 0; k < CW; ++k) v[k] = 0;
             const int nsrc = nsub + (sg > 0 ? 1 : 0);
@@ -1338,7 +1338,12 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
 
 // POOL: the fused 2x2/2 max-pool epilogue (a separate instantiation, so the
 // plain kernel carries none of its registers).
-template <int BITS, int NT, bool POOL>
+// LEAN: only the hot paths of the common plans (converter fast path, resident
+// filters in one slab, one accumulator group of at most two buffers, NT = 64).
+// Each SM sub-partition runs four warps of different roles from this one
+// kernel, and the general kernel's code for every other plan stalls their
+// instruction fetch: the benchmark layer runs ~9 % faster on the lean build.
+template <int BITS, int NT, bool POOL, bool LEAN>
 __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
 {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -1387,9 +1392,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
     const uint32_t tmem_base = *tmem_slot;
 
     if (warp < kConvWarps) {
-        converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty, stage_info);
+        converter_role<BITS, LEAN>(a, smem, raw_full, raw_empty, a_full, a_empty, stage_info);
     } else if (warp < kConvWarps + kEpiWarps) {
-        epilogue_role<BITS, NT, POOL>(a, smem, tmem_base, acc_full, acc_empty);
+        epilogue_role<BITS, NT, POOL, LEAN>(a, smem, tmem_base, acc_full, acc_empty);
     } else if (warp == kMmaWarp || (warp == kMmaWarp2 && a.mma_warps == 2)) {
         // the instruction descriptor is the same for both kinds (format fields 0: f16 / e4m3)
         const uint32_t idesc = idesc_f16_f32(kTileM, NT);
@@ -1404,7 +1409,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
                 else if (a.b_resident && a.nslab == 1 && ks == 2)
                     mma_role_resident<2, true>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full,
                                                acc_empty, done, stage_info, idesc, NT, sel, a.mma_warps);
-                else
+                else if (!LEAN)
                     mma_role<true>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
                                    stage_info, idesc, NT);
                 issued = true;
@@ -1420,7 +1425,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
         else if (a.b_resident && a.nslab == 1)
             mma_role_resident<1, false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
                                         stage_info, idesc, NT, sel, a.mma_warps);
-        else
+        else if (!LEAN)
             mma_role<false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done, stage_info,
                             idesc, NT);
     } else if (warp == kRawWarp) {
@@ -1582,13 +1587,13 @@ __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, con
     }
 }
 
-template <int BITS, int NT, bool POOL>
+template <int BITS, int NT, bool POOL, bool LEAN = false>
 cudaError_t launch_tc(const TcArgs &args, int grid, uint32_t smem, cudaStream_t st, bool after_prep)
 {
     // the opt-in shared-memory limit is raised once per device, outside any stream capture
     static std::mutex mu;
     static bool raised[64] = {};
-    auto kern = conv_tc_kernel<BITS, NT, POOL>;
+    auto kern = conv_tc_kernel<BITS, NT, POOL, LEAN>;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -1628,8 +1633,15 @@ cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, 
                                   : launch_tc<BITS, 16, false>(args, grid, smem, st, after_prep);
         case 32: return args.pool ? launch_tc<BITS, 32, true>(args, grid, smem, st, after_prep)
                                   : launch_tc<BITS, 32, false>(args, grid, smem, st, after_prep);
-        case 64: return args.pool ? launch_tc<BITS, 64, true>(args, grid, smem, st, after_prep)
-                                  : launch_tc<BITS, 64, false>(args, grid, smem, st, after_prep);
+        case 64: {
+            // the lean kernel serves plans whose every path it compiles (see conv_tc_kernel)
+            const bool lean = args.conv_fast && args.b_resident && args.nslab == 1 && args.nsg == 1 && args.nchunks <= 2;
+            if (lean)
+                return args.pool ? launch_tc<BITS, 64, true, true>(args, grid, smem, st, after_prep)
+                                 : launch_tc<BITS, 64, false, true>(args, grid, smem, st, after_prep);
+            return args.pool ? launch_tc<BITS, 64, true>(args, grid, smem, st, after_prep)
+                             : launch_tc<BITS, 64, false>(args, grid, smem, st, after_prep);
+        }
         case 128: return args.pool ? launch_tc<BITS, 128, true>(args, grid, smem, st, after_prep)
                                    : launch_tc<BITS, 128, false>(args, grid, smem, st, after_prep);
         default: return cudaErrorInvalidValue;
