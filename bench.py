@@ -332,7 +332,7 @@ def run_ours(args, world, rank, local):
                        "timing": "CUDA graphs of qconv_hwc calls, CUDA events on the launching stream"},
             "gpu_launches": launches_per_step * k,
             "roofline": {
-                "kernel": "conv_tc_kernel<8,64,false>",
+                "kernel": "conv_tc_kernel<8,64,false,2>",
                 "bound": "tensor",
                 "achieved": round(achieved_tflops, 1),
                 "peak": pk["bf16_tflops"],

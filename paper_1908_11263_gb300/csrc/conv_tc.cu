@@ -599,7 +599,7 @@ __device__ __forceinline__ void convert_fast(const TcArgs &a, const uint8_t *raw
     }
 }
 
-template <int BITS, bool LEAN>
+template <int BITS, int LEAN>
 __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
                                uint64_t *a_full, uint64_t *a_empty, volatile uint32_t *stage_info)
 {
@@ -631,7 +631,10 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
             uint8_t *st = smem + a.off_stages + stage * a.stage_bytes;
             bool staged = false;
-            if constexpr (BITS != 8) {
+            if constexpr (LEAN == 2) {  // row tiles, kernels at most 3 wide, fp16 staging
+                convert_fast<BITS, 3, false, false>(a, raw, st, g, item, mp, slab);
+                staged = true;
+            } else if constexpr (BITS != 8) {
                 if (a.fp8) {  // always on the fast path (planner)
                     if (a.strip)
                         convert_fast<BITS, 1, true, true>(a, raw, st, g, item, mp, slab);
@@ -1160,7 +1163,7 @@ __device__ __forceinline__ void release_acc(uint64_t *bar)
 // back and releases the group before the compression arithmetic, so the MMA
 // warp can refill it meanwhile.  Tiles that take several groups carry their
 // running sums in TMEM.
-template <int BITS, int NT, bool POOL, bool LEAN>
+template <int BITS, int NT, bool POOL, int LEAN>
 __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, uint32_t tmem_base, uint64_t *acc_full,
                                               uint64_t *acc_empty)
 {
@@ -1338,12 +1341,13 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
 
 // POOL: the fused 2x2/2 max-pool epilogue (a separate instantiation, so the
 // plain kernel carries none of its registers).
-// LEAN: only the hot paths of the common plans (converter fast path, resident
-// filters in one slab, one accumulator group of at most two buffers, NT = 64).
-// Each SM sub-partition runs four warps of different roles from this one
-// kernel, and the general kernel's code for every other plan stalls their
-// instruction fetch: the benchmark layer runs ~9 % faster on the lean build.
-template <int BITS, int NT, bool POOL, bool LEAN>
+// LEAN 1: only the hot paths of the common plans (converter fast path,
+// resident filters in one slab, one accumulator group of at most two buffers,
+// NT = 64).  LEAN 2: of those, only row tiles of kernels at most 3 wide with
+// fp16 staging and two k-steps per tap (INT-8, 32 channels per tap).  Each SM
+// sub-partition runs four warps of different roles from this one kernel, and
+// code for other plans stalls their instruction fetch.
+template <int BITS, int NT, bool POOL, int LEAN>
 __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
 {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -1401,7 +1405,11 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
         const int sel = warp == kMmaWarp ? 0 : 1;
         const int ks = a.cs / (2 * a.kch);  // k-steps per tap and slab
         bool issued = false;
-        if constexpr (BITS != 8) {
+        if constexpr (LEAN == 2) {
+            mma_role_resident<2, false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
+                                        stage_info, idesc, NT, sel, a.mma_warps);
+            issued = true;
+        } else if constexpr (BITS != 8) {
             if (a.fp8) {
                 if (a.b_resident && a.nslab == 1 && ks == 1)
                     mma_role_resident<1, true>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full,
@@ -1587,7 +1595,7 @@ __global__ void __launch_bounds__(256) conv_tc_prep_kernel(const uint8_t *w, con
     }
 }
 
-template <int BITS, int NT, bool POOL, bool LEAN = false>
+template <int BITS, int NT, bool POOL, int LEAN = 0>
 cudaError_t launch_tc(const TcArgs &args, int grid, uint32_t smem, cudaStream_t st, bool after_prep)
 {
     // the opt-in shared-memory limit is raised once per device, outside any stream capture
@@ -1636,9 +1644,13 @@ cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, 
         case 64: {
             // the lean kernel serves plans whose every path it compiles (see conv_tc_kernel)
             const bool lean = args.conv_fast && args.b_resident && args.nslab == 1 && args.nsg == 1 && args.nchunks <= 2;
+            if constexpr (BITS == 8) {
+                if (lean && !args.pool && !args.strip && args.kw <= 3 && args.cs == 32)
+                    return launch_tc<BITS, 64, false, 2>(args, grid, smem, st, after_prep);
+            }
             if (lean)
-                return args.pool ? launch_tc<BITS, 64, true, true>(args, grid, smem, st, after_prep)
-                                 : launch_tc<BITS, 64, false, true>(args, grid, smem, st, after_prep);
+                return args.pool ? launch_tc<BITS, 64, true, 1>(args, grid, smem, st, after_prep)
+                                 : launch_tc<BITS, 64, false, 1>(args, grid, smem, st, after_prep);
             return args.pool ? launch_tc<BITS, 64, true>(args, grid, smem, st, after_prep)
                              : launch_tc<BITS, 64, false>(args, grid, smem, st, after_prep);
         }
