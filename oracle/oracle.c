@@ -10,7 +10,7 @@
  * way this code can differ from the mathematics is a logic error, which the
  * pins in tests/test_oracle_pins.py are written to catch.
  *
- * Readings of the paper that this file fixes (each also listed in the design doc):
+ * Readings of the paper that this file fixes:
  *  - Activations are unsigned Q-bit integers, weights signed two's-complement
  *    Q-bit integers (the paper's INT-Q representation, Sec. III-A, Eq. 1).
  *  - The accumulator is the integer sum of products Phi(W,X) (Sec. III-A, Eq. 2),
