@@ -110,6 +110,18 @@ def test_algo_selection_and_workspace(lib):
         qnn.conv_algo(desc(bits=5))
 
 
+def test_subbyte_layers_with_c_multiple_of_32_plan_e4m3_filters(lib):
+    """INT-4/INT-2 layers whose C is a multiple of 32 stage e4m3 bytes (one byte per filter
+    element in the workspace); INT-8 and C = 16 keep fp16 (two bytes). The workspace is the
+    filters plus 96 bytes of per-channel constants and thresholds."""
+    consts = 64 * (32 + 64)
+    assert qnn.workspace_size(desc()) == 64 * 3 * 3 * 32 * 2 + consts
+    for bits in (4, 2):
+        assert qnn.workspace_size(desc(bits=bits)) == 64 * 3 * 3 * 32 * 1 + consts
+        d16 = qnn.conv_desc(1, 8, 8, 16, 64, 3, 3, 1, 1, bits, 10)
+        assert qnn.workspace_size(d16) == 64 * 3 * 3 * 16 * 2 + consts
+
+
 def test_other_entry_points_validate(lib):
     P = ctypes.c_void_p
     assert lib.qlinear(-1, 4, 4, P(FAKE), P(FAKE), None, P(FAKE), None) == qnn.QNN_EINVAL
