@@ -631,8 +631,8 @@ __device__ __forceinline__ void converter_role(const TcArgs &a, uint8_t *smem, u
             if (!warp_wait(&a_empty[stage], a_ph ^ 1u, a.status)) return;
             uint8_t *st = smem + a.off_stages + stage * a.stage_bytes;
             bool staged = false;
-            if constexpr (LEAN == 2) {  // row tiles, kernels at most 3 wide, fp16 staging
-                convert_fast<BITS, 3, false, false>(a, raw, st, g, item, mp, slab);
+            if constexpr (LEAN == 2) {  // row tiles, kernels at most 3 wide; e4m3 staging below INT-8
+                convert_fast<BITS, 3, false, BITS != 8>(a, raw, st, g, item, mp, slab);
                 staged = true;
             } else if constexpr (BITS != 8) {
                 if (a.fp8) {  // always on the fast path (planner)
@@ -1344,7 +1344,8 @@ __device__ __forceinline__ void epilogue_role(const TcArgs &a, uint8_t *smem, ui
 // LEAN 1: only the hot paths of the common plans (converter fast path,
 // resident filters in one slab, one accumulator group of at most two buffers,
 // NT = 64).  LEAN 2: of those, only row tiles of kernels at most 3 wide with
-// fp16 staging and two k-steps per tap (INT-8, 32 channels per tap).  Each SM
+// 32 channels per tap: fp16 staging and two k-steps per tap at INT-8, e4m3
+// staging and one k-step per tap at INT-4/INT-2.  Each SM
 // sub-partition runs four warps of different roles from this one kernel, and
 // code for other plans stalls their instruction fetch.
 template <int BITS, int NT, bool POOL, int LEAN>
@@ -1406,8 +1407,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_tc_kernel(const TcArgs a)
         const int ks = a.cs / (2 * a.kch);  // k-steps per tap and slab
         bool issued = false;
         if constexpr (LEAN == 2) {
-            mma_role_resident<2, false>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty, acc_full, acc_empty, done,
-                                        stage_info, idesc, NT, sel, a.mma_warps);
+            mma_role_resident<BITS == 8 ? 2 : 1, BITS != 8>(a, smem, tmem_base, a_full, a_empty, b_full, b_empty,
+                                                            acc_full, acc_empty, done, stage_info, idesc, NT, sel,
+                                                            a.mma_warps);
             issued = true;
         } else if constexpr (BITS != 8) {
             if (a.fp8) {
@@ -1644,10 +1646,9 @@ cudaError_t launch_tc_bits(int nt, const TcArgs &args, int grid, uint32_t smem, 
         case 64: {
             // the lean kernel serves plans whose every path it compiles (see conv_tc_kernel)
             const bool lean = args.conv_fast && args.b_resident && args.nslab == 1 && args.nsg == 1 && args.nchunks <= 2;
-            if constexpr (BITS == 8) {
-                if (lean && !args.pool && !args.strip && args.kw <= 3 && args.cs == 32)
-                    return launch_tc<BITS, 64, false, 2>(args, grid, smem, st, after_prep);
-            }
+            // INT-8 with fp16 staging, or INT-4/INT-2 with e4m3 staging, at 32 channels per tap
+            if (lean && !args.pool && !args.strip && args.kw <= 3 && args.cs == 32 && (BITS == 8) == !args.fp8)
+                return launch_tc<BITS, 64, false, 2>(args, grid, smem, st, after_prep);
             if (lean)
                 return args.pool ? launch_tc<BITS, 64, true, 1>(args, grid, smem, st, after_prep)
                                  : launch_tc<BITS, 64, false, 1>(args, grid, smem, st, after_prep);
