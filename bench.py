@@ -375,15 +375,25 @@ def oracle_sample_rate(layer, ld, nimg, threads):
 
 
 def oracle_baseline(layer, ld, budget_s=15.0):
-    """The oracle as it stands, on all host cores, on a bounded batch sample."""
+    """The oracle as it stands, on all host cores, on a bounded sample of about budget_s seconds:
+    a batch prefix of the workload, or, when the whole batch takes less than half the budget,
+    the whole batch repeated to fill it."""
     threads = os.cpu_count() or 1
     probe = max(1, min(layer.n, threads))
     dt, macs = oracle_sample_rate(layer, ld, probe, threads)
     nimg = int(min(layer.n, max(probe, probe * budget_s / max(dt, 1e-6))))
     dt, macs = oracle_sample_rate(layer, ld, nimg, threads)
+    passes = 1
+    if nimg == layer.n and dt < budget_s / 2:
+        passes = max(1, int(budget_s / max(dt, 1e-6)))
+        dt, macs = 0.0, 0.0
+        for _ in range(passes):
+            d, m = oracle_sample_rate(layer, ld, nimg, threads)
+            dt += d
+            macs += m
     return {"value": round(macs / dt / 1e9, 3), "unit": "GMAC/s", "cores": threads, "kind": "oracle",
-            "sample": f"{nimg} of {layer.n} images of the workload ({macs / 1e9:.2f} GMAC, {dt:.1f} s, "
-                      f"OpenMP over images)"}
+            "sample": f"{nimg} of {layer.n} images of the workload x {passes} pass{'es' if passes > 1 else ''} "
+                      f"({macs / 1e9:.2f} GMAC, {dt:.1f} s, OpenMP over images)"}
 
 
 def run_reference(args, world, rank):
