@@ -251,6 +251,32 @@ def test_conv_pool2_against_independent_reference(bits):
     np.testing.assert_array_equal(got, want)
 
 
+@pytest.mark.parametrize("bits", [4, 2])
+def test_staircase_realises_batch_norm_then_quantisation(bits):
+    """Footnote to Eq. 3: the thresholds absorb the bias and batch normalisation
+    y = gamma/sigma * (b + phi - mu) + beta. For gamma > 0 and the Q-bit output floor(y) clipped to
+    [0, 2^Q - 1], the thresholds tau_p = ceil(mu - b + (p - beta) * sigma / gamma), p = 1 .. 2^Q - 1,
+    make the staircase count of Eq. 4 equal that output for every accumulator phi. The reference
+    side is exact rational arithmetic; accumulators around each threshold are included."""
+    g = np.random.default_rng(100 + bits)
+    top = (1 << bits) - 1
+    for _ in range(25):
+        gamma = Fraction(int(g.integers(1, 60)), int(g.integers(1, 60)))
+        sigma = Fraction(int(g.integers(1, 60)), int(g.integers(1, 20)))
+        beta = Fraction(int(g.integers(-60, 60)), 7)
+        mu = Fraction(int(g.integers(-900, 900)), 3)
+        b = int(g.integers(-300, 300))
+        tau = [math.ceil(mu - b + (p - beta) * sigma / gamma) for p in range(1, top + 1)]
+        assert tau == sorted(tau)
+        phis = set(range(-3000, 3000, 37))
+        for t in tau:
+            phis.update((t - 1, t, t + 1))
+        for phi in sorted(phis):
+            y = gamma / sigma * (b + phi - mu) + beta
+            want = min(max(math.floor(y), 0), top)
+            assert oracle.staircase(phi, tau, bits) == want, (phi, tau)
+
+
 def test_zero_weights_give_bias_only_output():
     n, h, w, c, m = 1, 4, 4, 8, 4
     x, _ = rand_layer(n, h, w, c, m, 3)
