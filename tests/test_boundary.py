@@ -4,6 +4,8 @@ launching anything (only argument checks run, no CUDA call is reached)."""
 import ctypes
 import os
 import re
+import shutil
+import subprocess
 
 import pytest
 
@@ -30,6 +32,15 @@ def test_header_declares_the_expected_surface():
     names = declared_functions()
     for f in ("qconv_hwc", "qlinear", "qmaxpool", "pack_subbyte", "unpack_subbyte", "qconv_hwc_workspace_size"):
         assert f in names
+
+
+def test_header_is_plain_c():
+    """The boundary is a C ABI: include/qnn.h compiles as pedantic C99 (no C++ or torch types)."""
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-fsyntax-only", "-x", "c", HEADER],
+                   check=True)
 
 
 def test_library_exports_every_declared_function(lib):
