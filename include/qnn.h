@@ -7,7 +7,9 @@
  * with 32-bit accumulation (Sec. III-B, Eq. 2 and Eq. 6), compression of the
  * accumulator back to Q bits (Sec. III-A), max-pooling and the fully connected
  * layer (Sec. IV-A), for INT-8 and packed INT-4 / INT-2 data (Sec. IV-A,
- * "Sub-byte Extensions").
+ * "Sub-byte Extensions").  Also: the staircase (threshold) compression of
+ * Eq. 4, the INT-1 XNOR / popcount convolution of Eq. 5, and a convolution
+ * with its 2x2 max-pooling fused into one kernel.
  *
  * Conventions shared by every entry point
  *  - Plain C types only.  Pointers marked "device" must point to memory of the
