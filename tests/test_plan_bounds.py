@@ -36,3 +36,20 @@ def test_plans_keep_every_access_in_bounds(tmp_path):
     text = out.stdout
     for word in ("strips", "rows", "e4m3", "fp16"):
         assert f" {word} " in text, word
+    # and the documented choices for the workloads' layers
+    plans = {line.split(": ok=")[0]: line.split(": ok=")[1] for line in text.splitlines() if ": ok=" in line}
+    expect = {
+        "512x16x16x32->64 k3x3 p1,1 q8 pool0": "rows fp16",    # whole output rows per row tile, kernel 3 wide
+        "512x16x16x32->64 k3x3 p1,1 q4 pool0": "rows e4m3",
+        "512x16x16x32->64 k3x3 p1,1 q2 pool0": "rows e4m3",
+        "64x56x56x64->64 k3x3 p1,1 q8 pool0": "strips fp16",
+        "64x28x28x128->128 k3x3 p1,1 q8 pool0": "strips fp16",
+        "64x14x14x256->256 k3x3 p1,1 q8 pool0": "strips fp16",
+        "64x14x14x256->512 k1x1 p0,0 q8 pool0": "rows fp16",   # a 1x1 kernel needs no copies
+        "1024x32x32x3->32 k5x5 p2,2 q8 pool0": "strips fp16",
+        "1024x16x16x32->32 k5x5 p2,2 q8 pool0": "strips fp16",
+        "1024x8x8x32->64 k5x5 p2,2 q8 pool0": "strips fp16",
+        "512x16x16x32->64 k3x3 p1,1 q8 pool1": "strips fp16",  # the fused pool always takes strips
+    }
+    for key, want in expect.items():
+        assert plans[key].split(" nt=")[0] == "1 " + want, (key, plans[key])
