@@ -7,9 +7,11 @@ preparation + implicit-GEMM convolution kernel).  Metric: GMAC/s.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
-Timing: W eager warm-up steps, then exactly K steps replayed from CUDA graphs,
-bracketed by a barrier and torch.cuda.synchronize() on both sides, timed with
-CUDA events on the launching stream; max over ranks.  Each step reads and
+Timing: W eager warm-up steps, then runs of exactly K steps replayed from CUDA
+graphs, back to back, each run timed with its own CUDA events on the launching
+stream, until at least 50 runs and one second are timed; the median run counts.
+All runs are bracketed by a barrier and torch.cuda.synchronize() on both sides;
+max over ranks.  Each step reads and
 writes its own buffer set, rotating over sets whose total exceeds the 129 MB
 L2, so every step streams its activations from HBM.
 
@@ -37,6 +39,11 @@ if ROOT not in sys.path:
 from paper_1908_11263_gb300 import inputs  # noqa: E402
 
 L2_BYTES = 129 * 1024 * 1024
+# timed runs of the k-step graph: at least this many, and at least this long in all
+MIN_REPLAYS, MIN_TIMED_SECONDS, MAX_REPLAYS = 50, 1.0, 20000
+# nominal dense-rate ratio of e4m3 (kind::f8f6f4) to fp16 (kind::f16) tensor-core MMAs;
+# only the bf16 rate is measured, so the e4m3 roof is that rate scaled by this ratio
+E4M3_PER_FP16 = 2.0
 WORKLOAD = "conv3x3_16x16x32_to_64_int8_n512"
 INT8_IMMA_TOPS = 151.6
 # 32-bit population counts per second on this GPU (all SMs; measured, 15.1 per SM per cycle at
@@ -220,26 +227,46 @@ def run_ours(args, world, rank, local):
                     fn(offset + i)
         return g
 
-    def timed(fn, k, bulk=False):
+    def timed(fn, k, bulk=False, min_reps=MIN_REPLAYS, min_seconds=MIN_TIMED_SECONDS):
+        """Median time of one run of exactly k steps.  The k steps are captured once
+        (graphs of at most 1000 steps) and the whole k-step run is replayed back to
+        back, each run bracketed by its own pair of CUDA events on the launching
+        stream, until at least min_reps runs and min_seconds have been timed; the
+        median run is returned (seconds) with the number of runs."""
         chunk = min(k, 1000)
         full, rem = divmod(k, chunk)
         g_full = capture(fn, chunk, 0, bulk)
         g_rem = capture(fn, rem, chunk, bulk) if rem else None
-        g_full.replay()  # settle
-        torch.cuda.synchronize(dev)
-        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        barrier(world)
-        torch.cuda.synchronize(dev)
-        with torch.cuda.stream(stream):
-            start.record(stream)
+
+        def run():
             for _ in range(full):
                 g_full.replay()
             if g_rem is not None:
                 g_rem.replay()
-            end.record(stream)
+
+        run()  # settle
+        torch.cuda.synchronize(dev)
+        # a first timed run sizes the repetition count
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            run()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        one = max(e0.elapsed_time(e1) / 1e3, 1e-7)
+        reps = int(min(MAX_REPLAYS, max(min_reps, math.ceil(min_seconds / one))))
+        events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        with torch.cuda.stream(stream):
+            for a, b in events:
+                a.record(stream)
+                run()
+                b.record(stream)
         torch.cuda.synchronize(dev)
         barrier(world)
-        return start.elapsed_time(end) / 1e3  # seconds
+        times = [a.elapsed_time(b) / 1e3 for a, b in events]
+        return statistics.median(times), reps
 
     k = args.steps
     try:
@@ -247,8 +274,8 @@ def run_ours(args, world, rank, local):
     except Exception:
         gpu_id = str(local)
     with ClockSampler(gpu_id) as clk:
-        t_step = timed(step, k)
-        t_kernel = timed(kernel_only, k)
+        t_step, reps = timed(step, k)
+        t_kernel, _ = timed(kernel_only, k)
     qnn.device_status(stream)
     t_max = max_over_ranks(t_step, world, dev)
     clocks = clk.summary()
@@ -295,7 +322,7 @@ def run_ours(args, world, rank, local):
     with torch.cuda.stream(stream):
         e2e_steps(0, 3)
     e2e_k = max(10, min(k, 2000))
-    t_e2e = max_over_ranks(timed(e2e_steps, e2e_k, bulk=True), world, dev)
+    t_e2e = max_over_ranks(timed(e2e_steps, e2e_k, bulk=True, min_reps=5, min_seconds=0.05)[0], world, dev)
 
     # parity spot-check of the last output set against a second, independent GPU kernel
     ref = qnn.conv_hwc(xs[0], w, kappa, lam, bias=bias, shift=ld.shift, bits=8, stride=1, pad=1,
@@ -329,7 +356,8 @@ def run_ours(args, world, rank, local):
                        "filters": [layer.m, layer.k, layer.k, layer.c], "stride": 1, "pad": 1, "bits": 8,
                        "shift": ld.shift, "parallelism": f"replicas x{world}",
                        "l2": f"rotating {nsets} buffer sets ({nsets * per_set / 2**20:.0f} MiB > L2)",
-                       "timing": "CUDA graphs of qconv_hwc calls, CUDA events on the launching stream"},
+                       "timing": f"median of {reps} back-to-back runs of exactly {k} steps (CUDA graphs of "
+                                 f"qconv_hwc calls), each run timed with CUDA events on the launching stream"},
             "gpu_launches": launches_per_step * k,
             "roofline": {
                 "kernel": "conv_tc_kernel<8,64,false,2>",
@@ -355,6 +383,9 @@ def run_ours(args, world, rank, local):
                     "pipeline": "input copy, compute and output copy of consecutive steps on three streams"},
             "clocks": clocks,
         }
+        if clocks and clocks.get("sm_mhz"):
+            # clock-normalised step time: compare runs taken at different SM clocks
+            clocks["step_us_x_sm_mhz"] = round(t_max / k * 1e6 * clocks["sm_mhz"], 1)
         if args.cpu_baseline:
             result["cpu_baseline"] = oracle_baseline(layer, ld, budget_s=args.cpu_seconds)
     return result
@@ -442,7 +473,7 @@ def run_reference(args, world, rank):
 # ---------------------------------------------------------------------------- per-config sweep
 
 def run_sweep(args):
-    """One JSON line per layer of workloads 1, 3, 4 and 5 (workload 2 is the default run):
+    """One JSON line per layer of workloads 1 to 5:
     GMAC/s of qconv_hwc calls and of the convolution kernel alone, each timed from CUDA
     graphs over rotating buffer sets larger than L2, with the roof that binds the layer
     (its arithmetic intensity against the measured ridge) and the fraction reached."""
@@ -452,7 +483,6 @@ def run_sweep(args):
     torch.cuda.set_device(dev)
     qnn.load(build_if_missing=True)
     pk = peaks()
-    ridge = pk["bf16_tflops"] * 1e12 / (pk["hbm_gbs"] * 1e9)
     stream = torch.cuda.Stream(device=dev)
 
     def dev_packed(vals, bits, shape_bytes):
@@ -490,14 +520,50 @@ def run_sweep(args):
             t["x"] = dev_packed(ld.x, layer.bits, (layer.n, layer.h, layer.w, layer.c // per))
         return ld, t
 
-    def roof(flops, nbytes, seconds):
+    def roof(flops, nbytes, seconds, operand_bits=16):
+        """The binding roof of a layer: tensor when its arithmetic intensity exceeds the ridge
+        of the tensor rate its MMAs run at (fp16, or e4m3 at the nominal 2x the measured
+        bf16/fp16 rate), else HBM."""
+        scale = E4M3_PER_FP16 if operand_bits == 8 else 1.0
+        tpeak = pk["bf16_tflops"] * scale
         ai = flops / nbytes
-        if ai >= ridge:
-            return {"bound": "tensor", "achieved": round(flops / seconds / 1e12, 1), "peak": pk["bf16_tflops"],
-                    "unit": "TFLOP/s", "frac": round(flops / seconds / 1e12 / pk["bf16_tflops"], 4),
-                    "arith_intensity": round(ai, 1)}
+        if ai >= tpeak * 1e12 / (pk["hbm_gbs"] * 1e9):
+            src = (f"{pk['source']} bf16 dense burst x {E4M3_PER_FP16:g} (nominal e4m3:fp16 rate ratio; "
+                   f"kind::f8f6f4 MMAs)" if operand_bits == 8 else
+                   f"{pk['source']} bf16 dense burst (fp16 kind::f16 MMAs, same nominal rate)")
+            return {"bound": "tensor", "achieved": round(flops / seconds / 1e12, 1), "peak": round(tpeak, 1),
+                    "unit": "TFLOP/s", "frac": round(flops / seconds / 1e12 / tpeak, 4),
+                    "arith_intensity": round(ai, 1), "peak_source": src}
         return {"bound": "hbm", "achieved": round(nbytes / seconds / 1e9, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": round(nbytes / seconds / 1e9 / pk["hbm_gbs"], 4), "arith_intensity": round(ai, 1)}
+                "frac": round(nbytes / seconds / 1e9 / pk["hbm_gbs"], 4), "arith_intensity": round(ai, 1),
+                "peak_source": f"{pk['source']} HBM copy bandwidth"}
+
+    def oracle_times(layer, ld):
+        """The oracle on this layer: one thread on a batch prefix of about 1.5 s, scaled to the
+        whole batch, and all host cores on the whole batch (OpenMP over images)."""
+        import oracle
+        if not args.oracle_times:
+            return None
+        per = 8 // layer.bits
+        xs = ld.x.reshape(layer.n, -1)
+        wp = ld.w.reshape(-1).astype(np.int8).view(np.uint8) if layer.bits == 8 else oracle.pack(ld.w.reshape(-1), layer.bits)
+        threads = os.cpu_count() or 1
+
+        def run(nimg, nth):
+            shape = layer.shape()
+            shape["n"] = nimg
+            xi = xs[:nimg].reshape(-1)
+            xp = xi.astype(np.uint8) if layer.bits == 8 else oracle.pack(xi, layer.bits)
+            t0 = time.perf_counter()
+            oracle.conv_hwc(xp, wp, shape, ld.bias, ld.kappa, ld.lam, shifts=ld.shifts, shift=ld.shift, nthreads=nth)
+            return time.perf_counter() - t0
+
+        t1 = run(1, 1)
+        n1 = int(max(1, min(layer.n, 1.5 / max(t1, 1e-6))))
+        t1 = run(n1, 1) * layer.n / n1
+        tall = run(layer.n, threads)
+        return {"one_thread_s": round(t1, 4), "one_thread_sample": f"{n1} of {layer.n} images, scaled",
+                "all_cores_s": round(tall, 4), "cores": threads, "per_image_bytes": layer.h * layer.w * layer.c // per}
 
     def conv_line(config, key, layer, wl, lid, extra=None):
         ld, t = layer_tensors(key, layer, wl, lid)
@@ -532,11 +598,14 @@ def run_sweep(args):
             t_kernel = graph_time(lambda i: prepared(xs[i % nsets], out=ys[i % nsets], stream=stream), count, 3)
         qnn.device_status(stream)
         tk = t_kernel if t_kernel is not None else t_call
+        opbits = qnn.mma_operand_bits(desc)
         line = {"sweep": config, "layer": layer.name, "algo": "tensorcore" if algo == qnn.ALGO_TENSORCORE else "direct",
+                "mma_operands": {16: "fp16", 8: "e4m3", 0: "none (CUDA cores)"}[opbits],
                 "macs": layer.macs, "gmacs_call": round(layer.macs / t_call / 1e9, 1), "us_call": round(t_call * 1e6, 3),
                 "gmacs_kernel": round(layer.macs / tk / 1e9, 1), "us_kernel": round(tk * 1e6, 3),
-                "algorithmic_bytes": layer.algorithmic_bytes(), "roofline": roof(2.0 * layer.macs, layer.algorithmic_bytes(), tk),
-                "l2": f"rotating {nsets} buffer sets"}
+                "algorithmic_bytes": layer.algorithmic_bytes(),
+                "roofline": roof(2.0 * layer.macs, layer.algorithmic_bytes(), tk, opbits),
+                "oracle": oracle_times(layer, ld), "l2": f"rotating {nsets} buffer sets"}
         if extra:
             line.update(extra)
         print(json.dumps(line), flush=True)
@@ -563,6 +632,9 @@ def run_sweep(args):
     print(json.dumps({"sweep": "1", "layer": layer.name, "us_call_graph": round(t_graph * 1e6, 3),
                       "us_call_plain_launch": round(t_plain * 1e6, 3)}), flush=True)
 
+    # config 2: the default run's layer, here with the same per-layer columns as the others
+    (key, layer, wl, lid), = inputs.single_layer_workload(inputs.WORKLOAD_BATCH)
+    conv_line("2", key, layer, wl, lid)
     # config 4: INT-4 and INT-2
     for key, layer, wl, lid in inputs.single_layer_workload(inputs.WORKLOAD_SUBBYTE):
         conv_line("4", key, layer, wl, lid)
@@ -696,12 +768,14 @@ def run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=100000)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--sweep", action="store_true", help="per-config measurement lines (workloads 1, 3, 4, 5)")
+    ap.add_argument("--no-oracle-times", dest="oracle_times", action="store_false",
+                    help="--sweep without the oracle's one-thread and all-core times per layer")
     args = ap.parse_args()
     if args.sweep:
         run_sweep(args)

@@ -203,6 +203,15 @@ qnn_status qconv_hwc_binary(const qnn_conv_desc *d, const void *x, const void *w
  * negative qnn_status on invalid or unsupported descriptors. */
 int32_t qconv_hwc_algo(const qnn_conv_desc *d);
 
+/* Operand format of the tensor-core MMAs qconv_hwc() would issue for d, so that a
+ * caller can take the right tensor roof: 16 for fp16 operands (tcgen05 kind::f16,
+ * the exact embedding of INT-8 and of sub-byte layers with c not a multiple of 32),
+ * 8 for e4m3 operands (kind::f8f6f4, twice the fp16 rate per MMA; INT-4/INT-2 with
+ * c a multiple of 32), 0 when d selects the CUDA-core kernel; negative qnn_status
+ * on invalid or unsupported descriptors.  Not a paper concept: a query about this
+ * library's kernel choice. */
+int32_t qconv_hwc_mma_operand_bits(const qnn_conv_desc *d);
+
 /* Size of the fixed scratch array behind qconv_hwc_noalloc(): 2 MiB. */
 enum { QNN_NOALLOC_SCRATCH_BYTES = 2097152 };
 
@@ -237,6 +246,8 @@ enum { QNN_NOALLOC_SCRATCH_BYTES = 2097152 };
  *    calls.  Calls that overlap on the GPU (streams with no ordering between
  *    them) race on the array and give undefined results; calls queued on one
  *    stream do not overlap.
+ *  - n == 0: after validation, returns QNN_OK with nothing enqueued (the
+ *    scratch array is not touched).
  */
 qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *bias,
                              const int16_t *kappa, const int32_t *lambda, const uint8_t *shifts, void *y,

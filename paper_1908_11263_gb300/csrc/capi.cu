@@ -174,6 +174,18 @@ int32_t qconv_hwc_algo(const qnn_conv_desc *d)
     return choose_algo(d, s, &plan);
 }
 
+int32_t qconv_hwc_mma_operand_bits(const qnn_conv_desc *d)
+{
+    ConvShape s;
+    qnn_status st = check_conv(d, &s);
+    if (st != QNN_OK) return -static_cast<int32_t>(st);
+    TcPlan plan;
+    const int algo = choose_algo(d, s, &plan);
+    if (algo < 0) return algo;
+    if (algo != QNN_ALGO_TENSORCORE) return 0;
+    return plan.fp8 ? 8 : 16;
+}
+
 qnn_status qconv_hwc_prepare(const qnn_conv_desc *d, const void *w, const int32_t *bias, const int16_t *kappa,
                              const int32_t *lambda, const uint8_t *shifts, void *workspace, size_t workspace_bytes,
                              void *stream)
@@ -326,6 +338,9 @@ qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *
     if (st != QNN_OK) return st;
     if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE) return QNN_EUNSUPPORTED;
     if (plan.workspace_bytes > static_cast<size_t>(QNN_NOALLOC_SCRATCH_BYTES)) return QNN_ESCRATCH;
+    // an empty batch computes nothing, so it enqueues nothing and leaves the
+    // shared scratch array to the calls that use it
+    if (s.n == 0) return QNN_OK;
     void *scratch = noalloc_scratch_ptr();
     if (!scratch) return QNN_ECUDA;
     // the prep kernel rewrites every scratch byte the convolution reads, so the

@@ -41,13 +41,16 @@
 // copies.  Accumulators form a ring of up to four TMEM buffers, so the MMAs of
 // the next tile run while the epilogue compresses the current one.
 //
-// Warp roles (one persistent CTA per SM, 11 warps):
-//   warps 0-3  converters: raw u8 window -> fp16 copies
-//   warps 4-7  epilogue: TMEM -> registers, integer sum of chunks, compression,
-//              Q-bit packing, store
-//   warp 8     MMA issue (the warp runs converged; lane 0 issues tcgen05.mma)
-//   warp 9     bulk copies of input rows (lane 0 issues)
-//   warp 10    bulk copies of filters (lane 0 issues)
+// Warp roles (one persistent CTA per SM, 16 warps):
+//   warps 0-3   converters: raw window -> staged fp16 (or e4m3) operand
+//   warps 4-11  epilogue, two per TMEM lane quarter (one per column half):
+//               TMEM -> registers, integer sum of chunks, compression, Q-bit
+//               packing, store
+//   warp 12     MMA issue (the warp runs converged; an elected lane issues)
+//   warp 13     bulk copies of input rows (lane 0 issues)
+//   warp 14     bulk copies of filters (lane 0 issues)
+//   warp 15     second MMA issuer, taking alternate tiles, when one resident
+//               filter set serves the whole kernel
 // Every wait is bounded; on a timeout the kernel records QNN_ETIMEOUT in the
 // status word, stops its work, lets its copies and MMAs drain and frees TMEM.
 #include <cuda_fp16.h>

@@ -26,7 +26,8 @@ ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
             "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
-            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary", "qconv_hwc_pool2")
+            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary", "qconv_hwc_pool2",
+            "qconv_hwc_mma_operand_bits")
 
 
 class QnnError(RuntimeError):
@@ -80,6 +81,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_thresholds.restype = I32
         lib.qconv_hwc_noalloc.restype = I32
         lib.qconv_hwc_algo.restype = I32
+        lib.qconv_hwc_mma_operand_bits.argtypes = [DP]
+        lib.qconv_hwc_mma_operand_bits.restype = I32
         lib.qlinear.argtypes = [I32, I32, I32, P, P, P, P, P]
         lib.qlinear.restype = I32
         lib.qmaxpool.argtypes = [I32] * 7 + [P, P, P]
@@ -148,6 +151,15 @@ def conv_algo(desc: ConvDesc) -> int:
     r = load().qconv_hwc_algo(ctypes.byref(desc))
     if r < 0:
         raise QnnError(-r, "qconv_hwc_algo")
+    return r
+
+
+def mma_operand_bits(desc: ConvDesc) -> int:
+    """Operand width of the tensor-core MMAs for this descriptor: 16 (fp16, kind::f16),
+    8 (e4m3, kind::f8f6f4) or 0 (CUDA-core kernel)."""
+    r = load().qconv_hwc_mma_operand_bits(ctypes.byref(desc))
+    if r < 0:
+        raise QnnError(-r, "qconv_hwc_mma_operand_bits")
     return r
 
 

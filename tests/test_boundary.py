@@ -131,6 +131,13 @@ def test_subbyte_layers_with_c_multiple_of_32_plan_e4m3_filters(lib):
         assert qnn.workspace_size(desc(bits=bits)) == 64 * 3 * 3 * 32 * 1 + consts
         d16 = qnn.conv_desc(1, 8, 8, 16, 64, 3, 3, 1, 1, bits, 10)
         assert qnn.workspace_size(d16) == 64 * 3 * 3 * 16 * 2 + consts
+        # the operand-format query agrees: e4m3 (8 bits) with C = 32, fp16 with C = 16
+        assert qnn.mma_operand_bits(desc(bits=bits)) == 8
+        assert qnn.mma_operand_bits(d16) == 16
+    assert qnn.mma_operand_bits(desc()) == 16
+    assert qnn.mma_operand_bits(desc(stride=(2, 2))) == 0
+    with pytest.raises(qnn.QnnError):
+        qnn.mma_operand_bits(desc(bits=5))
 
 
 def test_other_entry_points_validate(lib):

@@ -108,6 +108,33 @@ def test_conv_pool2_equals_conv_then_qmaxpool_on_gpu():
     torch.cuda.synchronize()
     assert torch.equal(fused, two_step)
 
+@pytest.mark.gpu
+def test_conv_pool2_cifar_chain_batch1024():
+    """The CIFAR-10-shaped network of Sec. V-E at batch 1024, run as the benchmark runs it: each
+    convolution with its 2x2 max-pool fused (qconv_hwc_pool2), chained on the device, then the
+    fully connected layer.  Every pooled activation and every FC output is compared with the
+    oracle's chain (conv_hwc then maxpool per layer, then linear)."""
+    from paper_1908_11263_gb300 import inputs
+    n = 1024
+    x = inputs.cifar_input(n)
+    xd = to_dev(x.astype(np.uint8))
+    xo = x.astype(np.uint8).reshape(-1)
+    for key, layer, wl, lid in inputs.cifar_layers(n):
+        ld = inputs.make_layer(key, layer, wl, lid, x=np.zeros(1))
+        yd = qnn.conv_hwc_pool2(xd, to_dev(ld.w), to_dev(ld.kappa, torch.int16), to_dev(ld.lam, torch.int32),
+                                bias=to_dev(ld.bias, torch.int32), shift=ld.shift, bits=8, pad=layer.pad)
+        qnn.device_status()
+        yo = oracle.conv_hwc_pool2(xo, ld.w.reshape(-1).view(np.uint8), layer.shape(), ld.bias, ld.kappa, ld.lam,
+                                   shift=ld.shift, nthreads=THREADS)
+        got = yd.cpu().numpy().reshape(-1)
+        assert first_mismatch(got, yo) is None, (key, first_mismatch(got, yo))
+        assert len(np.unique(yo)) > 16, f"{key}: pooled outputs nearly constant, the check is weak"
+        xd, xo = yd, yo
+    wfc, bfc = inputs.cifar_fc()
+    yd = qnn.linear(xd.view(n, -1), to_dev(wfc), to_dev(bfc))
+    yo = oracle.linear(xo.reshape(n, -1), wfc, bfc)
+    np.testing.assert_array_equal(yd.cpu().numpy(), yo)
+
 
 @pytest.fixture(scope="module")
 def lib():

@@ -106,6 +106,33 @@ def test_noalloc_matches_qconv_hwc_on_consecutive_calls():
             assert bool((buf[-GUARD:] == 0xA5).all()), f"layer {i}: write past the end of the output"
 
 
+@pytest.mark.gpu
+def test_noalloc_allocates_no_device_memory():
+    """The property the entry point exists for: once each layer has run once on the
+    device (set-up done), further calls take no device memory, neither from the CUDA
+    driver (free memory does not drop) nor from torch's caching allocator (its
+    allocated bytes stay the same; the outputs are allocated before the count)."""
+    layers = [_layer(**spec) for spec in LAYERS]
+    outs = [torch.empty(layer["out_shape"], dtype=torch.uint8, device="cuda:0") for layer in layers]
+
+    def run_all():
+        for layer, out in zip(layers, outs):
+            qnn.conv_hwc_noalloc(layer["x"], layer["w"], layer["kappa"], layer["lam"], out, bias=layer["bias"],
+                                 shifts=layer["shifts"], shift=layer["shift"], bits=layer["bits"], pad=layer["pad"])
+
+    run_all()  # first use on this device: set-up, and every kernel instantiation loaded
+    torch.cuda.synchronize()
+    free_before, _ = torch.cuda.mem_get_info()
+    allocated_before = torch.cuda.memory_allocated()
+    for _ in range(8):
+        run_all()
+    qnn.device_status()
+    torch.cuda.synchronize()
+    free_after, _ = torch.cuda.mem_get_info()
+    assert torch.cuda.memory_allocated() == allocated_before
+    assert free_after >= free_before, f"device free memory dropped by {free_before - free_after} bytes"
+
+
 @pytest.fixture(scope="module")
 def lib():
     qbuild.build()
@@ -129,3 +156,12 @@ def test_noalloc_rejects_what_it_cannot_run(lib):
     ok = qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 1, 1, 8, 10)
     assert status(ok, x=0) == qnn.QNN_EINVAL
     assert status(ok, y=FAKE + 8) == qnn.QNN_EALIGN
+
+
+def test_noalloc_empty_batch_enqueues_nothing(lib):
+    """n == 0 returns QNN_OK right after validation, before any CUDA call (so it also
+    runs without a GPU) and without touching the shared scratch array."""
+    P = ctypes.c_void_p
+    empty = qnn.conv_desc(0, 16, 16, 32, 64, 3, 3, 1, 1, 8, 12)
+    assert lib.qconv_hwc_noalloc(ctypes.byref(empty), None, P(FAKE), P(FAKE), P(FAKE), P(FAKE), None, None,
+                                 None) == qnn.QNN_OK
