@@ -52,8 +52,9 @@ POPC_TPS = 4.77
 METRIC = "qconv_hwc GMAC/s (16x16x32 -> 64, 3x3, stride 1, pad 1, INT-8, batch 512)"
 
 
-PROFILE = os.path.join(ROOT, "profiles", "conv_tc_kernel_conv3x3_16x16x32to64_int8_n512.md")
-KERNEL_SOURCES = ("conv_tc.cu", "device.cuh", "internal.h")
+PROFILE = os.path.join(ROOT, "profiles", "conv_win_kernel_conv3x3_16x16x32to64_int8_n512.md")
+KERNEL_SOURCES = ("conv_win.cuh", "conv_win_inst.cuh", "conv_common.cuh", "device.cuh", "internal.h")
+KERNEL_NAME = "conv_win_kernel<8,64,false>"
 
 
 def measured_traffic():
@@ -195,10 +196,10 @@ def run_ours(args, world, rank, local):
     ys = [torch.empty((layer.n, layer.oh, layer.ow, layer.m), dtype=torch.uint8, device=dev) for _ in range(nsets)]
     desc = qnn.conv_desc(layer.n, layer.h, layer.w, layer.c, layer.m, layer.k, layer.k, layer.stride, layer.pad, 8,
                          ld.shift)
-    assert qnn.conv_algo(desc) == qnn.ALGO_TENSORCORE
+    assert qnn.tc_kernel(desc) == qnn.ALGO_TC_WINDOW
     ws = torch.empty(qnn.workspace_size(desc), dtype=torch.uint8, device=dev)
     stream = torch.cuda.Stream(device=dev)
-    launches_per_step = 2  # filter preparation + convolution kernel
+    launches_per_step = 1  # the window kernel: filter re-layout, convolution and compression in one launch
 
     def step(i):
         qnn.conv_hwc(xs[i % nsets], w, kappa, lam, bias=bias, shift=ld.shift, bits=8, stride=1, pad=1,
@@ -360,7 +361,7 @@ def run_ours(args, world, rank, local):
                                  f"qconv_hwc calls), each run timed with CUDA events on the launching stream"},
             "gpu_launches": launches_per_step * k,
             "roofline": {
-                "kernel": "conv_tc_kernel<8,64,false,2>",
+                "kernel": KERNEL_NAME,
                 "bound": "tensor",
                 "achieved": round(achieved_tflops, 1),
                 "peak": pk["bf16_tflops"],
@@ -599,7 +600,9 @@ def run_sweep(args):
         qnn.device_status(stream)
         tk = t_kernel if t_kernel is not None else t_call
         opbits = qnn.mma_operand_bits(desc)
+        kernel = {qnn.ALGO_TC_WINDOW: "window", qnn.ALGO_TC_GENERAL: "general", 0: "direct"}[qnn.tc_kernel(desc)]
         line = {"sweep": config, "layer": layer.name, "algo": "tensorcore" if algo == qnn.ALGO_TENSORCORE else "direct",
+                "kernel": kernel,
                 "mma_operands": {16: "fp16", 8: "e4m3", 0: "none (CUDA cores)"}[opbits],
                 "macs": layer.macs, "gmacs_call": round(layer.macs / t_call / 1e9, 1), "us_call": round(t_call * 1e6, 3),
                 "gmacs_kernel": round(layer.macs / tk / 1e9, 1), "us_kernel": round(tk * 1e6, 3),

@@ -55,7 +55,13 @@ typedef enum {
 enum {
     QNN_ALGO_AUTO = 0,         /* tensor-core kernel when the shape allows it, else the CUDA-core kernel */
     QNN_ALGO_DIRECT = 1,       /* CUDA-core kernel (dp4a), any stride / padding */
-    QNN_ALGO_TENSORCORE = 2    /* tcgen05 implicit GEMM; QNN_EUNSUPPORTED when the shape does not fit it */
+    QNN_ALGO_TENSORCORE = 2,   /* tcgen05 implicit GEMM (the window kernel when its plan fits, else the
+                                  general one); QNN_EUNSUPPORTED when neither fits the shape */
+    QNN_ALGO_TC_WINDOW = 3,    /* the window kernel only: stride 1, m <= 128, INT-8 with c a multiple of 8
+                                  or INT-4/INT-2 with c a multiple of 32, c <= 64 (INT-8) or 128 (sub-byte),
+                                  kh, kw <= 8; one launch per call, filters read in place */
+    QNN_ALGO_TC_GENERAL = 4    /* the general tensor-core kernel only (filter preparation kernel plus
+                                  convolution kernel, any stride-1 shape with whole 16-byte input rows) */
 };
 
 /*
@@ -77,11 +83,15 @@ typedef struct {
 } qnn_conv_desc;
 
 /*
- * Bytes of device workspace qconv_hwc() needs for this layer (0 when the
- * chosen kernel needs none).  The workspace holds the filters re-laid out for
- * the tensor cores and the per-channel compression constants; it is rewritten
- * by every call, so one workspace must not be shared by calls that can run
- * concurrently.
+ * Bytes of device workspace for this layer: what qconv_hwc_prepare() writes
+ * and qconv_hwc_run() reads, and what qconv_hwc() needs on the general
+ * tensor-core kernel (0 for the CUDA-core kernel).  For the general kernel
+ * the workspace holds the filters re-laid out for the tensor cores and the
+ * per-channel compression constants, rewritten by every qconv_hwc() call, so
+ * one workspace must not be shared by calls that can run concurrently.  For
+ * the window kernel it holds copies of the packed filters, bias, kappa, lambda
+ * and shifts, written by qconv_hwc_prepare() only (qconv_hwc() reads the
+ * caller's buffers in place and leaves it alone).
  */
 qnn_status qconv_hwc_workspace_size(const qnn_conv_desc *d, size_t *bytes);
 
@@ -103,7 +113,10 @@ qnn_status qconv_hwc_workspace_size(const qnn_conv_desc *d, size_t *bytes);
  *   y       device, packed unsigned Q-bit NHWC output, 16-byte aligned
  *   workspace, workspace_bytes: device scratch of at least
  *           qconv_hwc_workspace_size() bytes, 256-byte aligned (may be NULL
- *           when that size is 0)
+ *           when that size is 0).  When the window kernel serves the layer
+ *           (qconv_hwc_tc_kernel() == QNN_ALGO_TC_WINDOW) the call is one
+ *           launch that reads w, bias, kappa, lambda and shifts in place and
+ *           the workspace is neither read nor written (it may be NULL).
  *
  * Requirements (else QNN_EUNSUPPORTED): c and m multiples of 8/Q, and
  * kh*kw*c*(2^Q-1)*2^(Q-1) < 2^30, so that the int32 accumulator of Eq. 2 cannot
@@ -202,6 +215,11 @@ qnn_status qconv_hwc_binary(const qnn_conv_desc *d, const void *x, const void *w
 /* Which kernel qconv_hwc() would run for d: QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE;
  * negative qnn_status on invalid or unsupported descriptors. */
 int32_t qconv_hwc_algo(const qnn_conv_desc *d);
+
+/* Which tensor-core kernel qconv_hwc() would run for d: QNN_ALGO_TC_WINDOW or
+ * QNN_ALGO_TC_GENERAL; 0 when d selects the CUDA-core kernel; negative qnn_status
+ * on invalid or unsupported descriptors. */
+int32_t qconv_hwc_tc_kernel(const qnn_conv_desc *d);
 
 /* Operand format of the tensor-core MMAs qconv_hwc() would issue for d, so that a
  * caller can take the right tensor roof: 16 for fp16 operands (tcgen05 kind::f16,

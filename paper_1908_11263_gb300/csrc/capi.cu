@@ -64,7 +64,7 @@ qnn_status check_conv(const qnn_conv_desc *d, ConvShape *s)
     if (d->n < 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->m <= 0 || d->kh <= 0 || d->kw <= 0) return QNN_EINVAL;
     if (d->stride_h <= 0 || d->stride_w <= 0 || d->pad_h < 0 || d->pad_w < 0) return QNN_EINVAL;
     if (d->h + 2 * d->pad_h < d->kh || d->w + 2 * d->pad_w < d->kw) return QNN_EINVAL;
-    if (d->algo < QNN_ALGO_AUTO || d->algo > QNN_ALGO_TENSORCORE) return QNN_EINVAL;
+    if (d->algo < QNN_ALGO_AUTO || d->algo > QNN_ALGO_TC_GENERAL) return QNN_EINVAL;
     if (!bits_ok(d->bits)) return QNN_EUNSUPPORTED;
     const int per = 8 / d->bits;
     if (d->c % per || d->m % per) return QNN_EUNSUPPORTED;
@@ -78,13 +78,42 @@ qnn_status check_conv(const qnn_conv_desc *d, ConvShape *s)
     return QNN_OK;
 }
 
-// QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE, or a negative status.
+// Which kernel serves a descriptor.  Tensor-core requests (QNN_ALGO_AUTO,
+// QNN_ALGO_TENSORCORE) take the window kernel when its plan fits the shape,
+// else the general tensor-core kernel; QNN_ALGO_TC_WINDOW and
+// QNN_ALGO_TC_GENERAL force one of them.
+enum Kernel { kDirect = 1, kWindow = 3, kGeneral = 4 };
+
+struct Choice {
+    int kernel;  // Kernel, or a negative qnn_status
+    TcPlan plan;
+    WinPlan wplan;
+};
+
+Choice choose(const qnn_conv_desc *d, const ConvShape &s)
+{
+    Choice c;
+    c.plan = plan_conv_tc(s);
+    c.wplan = plan_conv_win(s);
+    switch (d->algo) {
+        case QNN_ALGO_DIRECT: c.kernel = kDirect; break;
+        case QNN_ALGO_TC_WINDOW: c.kernel = c.wplan.ok ? kWindow : -QNN_EUNSUPPORTED; break;
+        case QNN_ALGO_TC_GENERAL: c.kernel = c.plan.ok ? kGeneral : -QNN_EUNSUPPORTED; break;
+        case QNN_ALGO_TENSORCORE:
+            c.kernel = c.wplan.ok ? kWindow : c.plan.ok ? kGeneral : -QNN_EUNSUPPORTED;
+            break;
+        default: c.kernel = c.wplan.ok ? kWindow : c.plan.ok ? kGeneral : kDirect; break;
+    }
+    return c;
+}
+
+// QNN_ALGO_DIRECT or QNN_ALGO_TENSORCORE (either tensor-core kernel), or a negative status.
 int choose_algo(const qnn_conv_desc *d, const ConvShape &s, TcPlan *plan)
 {
-    *plan = plan_conv_tc(s);
-    if (d->algo == QNN_ALGO_DIRECT) return QNN_ALGO_DIRECT;
-    if (d->algo == QNN_ALGO_TENSORCORE) return plan->ok ? QNN_ALGO_TENSORCORE : -QNN_EUNSUPPORTED;
-    return plan->ok ? QNN_ALGO_TENSORCORE : QNN_ALGO_DIRECT;
+    const Choice c = choose(d, s);
+    *plan = c.plan;
+    if (c.kernel < 0) return c.kernel;
+    return c.kernel == kDirect ? QNN_ALGO_DIRECT : QNN_ALGO_TENSORCORE;
 }
 
 qnn_status from_cuda(cudaError_t e) { return e == cudaSuccess ? QNN_OK : QNN_ECUDA; }
@@ -158,11 +187,20 @@ qnn_status qconv_hwc_workspace_size(const qnn_conv_desc *d, size_t *bytes)
     ConvShape s;
     qnn_status st = check_conv(d, &s);
     if (st != QNN_OK) return st;
-    TcPlan plan;
-    const int algo = choose_algo(d, s, &plan);
-    if (algo < 0) return static_cast<qnn_status>(-algo);
-    *bytes = algo == QNN_ALGO_TENSORCORE ? plan.workspace_bytes : 0;
+    const Choice c = choose(d, s);
+    if (c.kernel < 0) return static_cast<qnn_status>(-c.kernel);
+    *bytes = c.kernel == kWindow ? c.wplan.param_bytes : c.kernel == kGeneral ? c.plan.workspace_bytes : 0;
     return QNN_OK;
+}
+
+int32_t qconv_hwc_tc_kernel(const qnn_conv_desc *d)
+{
+    ConvShape s;
+    qnn_status st = check_conv(d, &s);
+    if (st != QNN_OK) return -static_cast<int32_t>(st);
+    const Choice c = choose(d, s);
+    if (c.kernel < 0) return c.kernel;
+    return c.kernel == kDirect ? 0 : c.kernel;
 }
 
 int32_t qconv_hwc_algo(const qnn_conv_desc *d)
@@ -179,11 +217,11 @@ int32_t qconv_hwc_mma_operand_bits(const qnn_conv_desc *d)
     ConvShape s;
     qnn_status st = check_conv(d, &s);
     if (st != QNN_OK) return -static_cast<int32_t>(st);
-    TcPlan plan;
-    const int algo = choose_algo(d, s, &plan);
-    if (algo < 0) return algo;
-    if (algo != QNN_ALGO_TENSORCORE) return 0;
-    return plan.fp8 ? 8 : 16;
+    const Choice c = choose(d, s);
+    if (c.kernel < 0) return c.kernel;
+    if (c.kernel == kWindow) return c.wplan.fp8 ? 8 : 16;
+    if (c.kernel == kGeneral) return c.plan.fp8 ? 8 : 16;
+    return 0;
 }
 
 qnn_status qconv_hwc_prepare(const qnn_conv_desc *d, const void *w, const int32_t *bias, const int16_t *kappa,
@@ -196,10 +234,15 @@ qnn_status qconv_hwc_prepare(const qnn_conv_desc *d, const void *w, const int32_
     TcPlan plan;
     st = check_params(d, s, w, bias, kappa, lambda, shifts, &plan);
     if (st != QNN_OK) return st;
-    if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE) return QNN_OK;
+    const Choice c = choose(d, s);
+    if (c.kernel == kDirect) return QNN_OK;
+    ConvParams p{nullptr, static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts, d->shift, nullptr};
+    if (c.kernel == kWindow) {
+        if (!workspace || workspace_bytes < c.wplan.param_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
+        return from_cuda(prepare_conv_win(c.wplan, s, p, workspace, static_cast<cudaStream_t>(stream)));
+    }
     st = check_workspace(plan, workspace, workspace_bytes);
     if (st != QNN_OK) return st;
-    ConvParams p{nullptr, static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts, d->shift, nullptr};
     return from_cuda(launch_conv_tc_prep(plan, s, p, workspace, static_cast<cudaStream_t>(stream)));
 }
 
@@ -211,13 +254,19 @@ qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const v
     if (st != QNN_OK) return st;
     if (s.n > 0 && (!x || !y)) return QNN_EINVAL;
     if (!aligned(x, 16) || !aligned(y, 16)) return QNN_EALIGN;
-    TcPlan plan;
-    const int algo = choose_algo(d, s, &plan);
-    if (algo < 0) return static_cast<qnn_status>(-algo);
-    if (algo != QNN_ALGO_TENSORCORE) return QNN_EUNSUPPORTED;
-    st = check_workspace(plan, workspace, workspace_bytes);
+    const Choice c = choose(d, s);
+    if (c.kernel < 0) return static_cast<qnn_status>(-c.kernel);
+    if (c.kernel == kDirect) return QNN_EUNSUPPORTED;
+    if (c.kernel == kWindow) {
+        if (!workspace || workspace_bytes < c.wplan.param_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
+        ConvParams p = win_prepared_params(c.wplan, workspace);
+        p.x = static_cast<const uint8_t *>(x);
+        p.y = static_cast<uint8_t *>(y);
+        return from_cuda(launch_conv_win(c.wplan, s, p, static_cast<cudaStream_t>(stream)));
+    }
+    st = check_workspace(c.plan, workspace, workspace_bytes);
     if (st != QNN_OK) return st;
-    return from_cuda(launch_conv_tc_run(plan, s, static_cast<const uint8_t *>(x), static_cast<uint8_t *>(y),
+    return from_cuda(launch_conv_tc_run(c.plan, s, static_cast<const uint8_t *>(x), static_cast<uint8_t *>(y),
                                         workspace, static_cast<cudaStream_t>(stream), false));
 }
 
@@ -233,9 +282,14 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
     TcPlan plan;
     st = check_params(d, s, w, bias, kappa, lambda, shifts, &plan);
     if (st != QNN_OK) return st;
-    const int algo = choose_algo(d, s, &plan);
+    const Choice c = choose(d, s);
     cudaStream_t cs = static_cast<cudaStream_t>(stream);
-    if (algo == QNN_ALGO_TENSORCORE) {
+    if (c.kernel == kWindow) {  // one launch; the filters are read where the caller keeps them
+        ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
+                     d->shift, static_cast<uint8_t *>(y)};
+        return from_cuda(launch_conv_win(c.wplan, s, p, cs));
+    }
+    if (c.kernel == kGeneral) {
         st = check_workspace(plan, workspace, workspace_bytes);
         if (st != QNN_OK) return st;
         ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
@@ -264,13 +318,15 @@ qnn_status qconv_hwc_pool2(const qnn_conv_desc *d, const void *x, const void *w,
     TcPlan plan;
     st = check_params(d, s, w, bias, kappa, lambda, shifts, &plan);
     if (st != QNN_OK) return st;
-    // the fused pool runs in the tensor-core kernel only (strip tiles)
-    if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE || !plan.strip) return QNN_EUNSUPPORTED;
-    st = check_workspace(plan, workspace, workspace_bytes);
-    if (st != QNN_OK) return st;
+    // the fused pool runs in the tensor-core kernels only (strip tiles)
+    const Choice c = choose(d, s);
     cudaStream_t cs = static_cast<cudaStream_t>(stream);
     ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts,
                  d->shift, static_cast<uint8_t *>(y)};
+    if (c.kernel == kWindow) return from_cuda(launch_conv_win(c.wplan, s, p, cs));
+    if (c.kernel != kGeneral || !plan.strip) return QNN_EUNSUPPORTED;
+    st = check_workspace(plan, workspace, workspace_bytes);
+    if (st != QNN_OK) return st;
     cudaError_t e = launch_conv_tc_prep(plan, s, p, workspace, cs);
     if (e == cudaSuccess) e = launch_conv_tc_run(plan, s, p.x, p.y, workspace, cs, true);
     return from_cuda(e);
@@ -290,9 +346,11 @@ qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const voi
     TcPlan plan;
     const int algo = choose_algo(d, s, &plan);
     if (algo < 0) return static_cast<qnn_status>(-algo);
+    const Choice c = choose(d, s);
     cudaStream_t cs = static_cast<cudaStream_t>(stream);
     ConvParams p{static_cast<const uint8_t *>(x), static_cast<const uint8_t *>(w), nullptr, nullptr, nullptr, nullptr,
                  0, static_cast<uint8_t *>(y), thresholds};
+    if (c.kernel == kWindow) return from_cuda(launch_conv_win(c.wplan, s, p, cs));
     if (algo == QNN_ALGO_TENSORCORE) {
         st = check_workspace(plan, workspace, workspace_bytes);
         if (st != QNN_OK) return st;
@@ -336,7 +394,9 @@ qnn_status qconv_hwc_noalloc(const qnn_conv_desc *d, const void *x, const void *
     TcPlan plan;
     st = check_params(d, s, w, bias, kappa, lambda, shifts, &plan);
     if (st != QNN_OK) return st;
-    if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE) return QNN_EUNSUPPORTED;
+    // this entry point runs the general tensor-core kernel, whose prepared filters go to the scratch array
+    if (choose_algo(d, s, &plan) != QNN_ALGO_TENSORCORE || !plan.ok || d->algo == QNN_ALGO_TC_WINDOW)
+        return QNN_EUNSUPPORTED;
     if (plan.workspace_bytes > static_cast<size_t>(QNN_NOALLOC_SCRATCH_BYTES)) return QNN_ESCRATCH;
     // an empty batch computes nothing, so it enqueues nothing and leaves the
     // shared scratch array to the calls that use it

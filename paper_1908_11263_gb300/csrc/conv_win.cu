@@ -1,0 +1,242 @@
+// Host side of the window kernel (conv_win.cuh): the planner, the launch and
+// the prepared-workspace layout.
+#include <algorithm>
+
+#include "conv_win.cuh"
+
+namespace qnn {
+
+namespace {
+
+uint32_t round_up(uint32_t v, uint32_t a) { return (v + a - 1) / a * a; }
+size_t round_up_sz(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Shared-memory bytes of the barriers and the words after them (see the kernel).
+constexpr uint32_t kBarBytes = (4 * win::kMaxStages + 2 * win::kMaxSlots + 2) * 8 + sizeof(win::Misc);
+
+// Strips per tile: two unless the image is at most 8 columns wide, or the
+// second strip of a tile would compute more than 15 % extra columns.
+int strips_per_tile(int ow)
+{
+    if (ow <= win::kCols) return 1;
+    const long long w1 = (ow + 7) / 8 * 8LL, w2 = (ow + 15) / 16 * 16LL;
+    return w2 * 100 <= w1 * 115 ? 2 : 1;
+}
+
+}  // namespace
+
+WinPlan plan_conv_win(const ConvShape &s)
+{
+    WinPlan p{};
+    p.ok = false;
+    if (s.sh != 1 || s.sw != 1 || s.oh <= 0 || s.ow <= 0 || s.n < 0) return p;
+    p.fp8 = s.bits != 8;
+    p.kch = p.fp8 ? 16 : 8;
+    // INT-8 in fp16 (whole 8-channel chunks), INT-4 / INT-2 in e4m3 (whole 32-channel pairs)
+    if (s.bits == 8 ? (s.c % 8 != 0) : (s.c % 32 != 0)) return p;
+    if (s.m > 128) return p;  // one filter set, all output channels in one MMA N
+    p.nt = s.m <= 32 ? 32 : s.m <= 64 ? 64 : 128;
+    p.c_pad = (s.c + 2 * p.kch - 1) / (2 * p.kch) * (2 * p.kch);
+    p.groups = p.c_pad / p.kch;
+    if (p.groups > 8) return p;  // the window holds every channel of a pixel
+    p.taps = s.kh * s.kw;
+    if (s.kh > 8 || s.kw > 8 || p.taps > win::kMaxTaps) return p;
+    p.ksteps = p.groups / 2;
+    const long long cb = static_cast<long long>(s.c) * s.bits / 8;
+    // worst-case exact chunks: products of at most max|staged x| * max|w| each,
+    // whole taps (c_pad products per accumulator per tap) per chunk
+    const long long max_prod = p.fp8 ? (s.bits == 4 ? 15 * 8 : 3 * 2) : 128 * 128;
+    const long long taps_per_chunk = ((1ll << 22) / max_prod) / p.c_pad;
+    if (taps_per_chunk < 1) return p;
+    p.nch_max = static_cast<int>((p.taps + taps_per_chunk - 1) / taps_per_chunk);
+    if (p.nch_max > 16) return p;
+    const int s_pref = strips_per_tile(s.ow);
+    for (int S : {s_pref, 3 - s_pref}) {
+        if (S * p.nch_max * p.nt > 512) continue;  // one slot of accumulators in TMEM
+        const int sp = win::kCols * S + s.kw - 1, wh = win::kRows + s.kh - 1;
+        if (wh * sp > win::kMaxKP * 128) continue;  // converter positions per thread
+        const int tiles_x = (s.ow + win::kCols * S - 1) / (win::kCols * S);
+        const bool full_rows = tiles_x == 1;
+        const long long row_bytes = s.w * cb;
+        uint32_t raw_row_bytes;
+        if (full_rows) {
+            if (row_bytes % 16 != 0 || row_bytes > (1 << 20)) continue;  // rows move as one bulk copy
+            raw_row_bytes = static_cast<uint32_t>(row_bytes);
+        } else {
+            if (cb % 16 != 0) continue;  // per-row copies start at any pixel
+            raw_row_bytes = round_up(static_cast<uint32_t>(std::min(sp, s.w) * cb), 16);
+        }
+        const uint32_t raw_bytes = round_up(static_cast<uint32_t>(std::min(wh, s.h)) * raw_row_bytes, 128);
+        if (raw_bytes >= (1u << 20)) continue;  // one transaction count
+        const uint32_t p_alloc = round_up(static_cast<uint32_t>(wh * sp), 8);
+        const uint32_t chunk_stride = p_alloc * 16;
+        const uint32_t stage_bytes = chunk_stride * p.groups;
+        const uint32_t b_bytes = static_cast<uint32_t>(p.taps * p.groups * p.nt * 16);
+        // rec0, rec1 (16 bytes each), compact direct constants (8), direct flags (1 per 16 channels)
+        const uint32_t rec_bytes = round_up(static_cast<uint32_t>(2 * p.nt * 16 + p.nt * 8 + p.nt / 16), 16);
+        const uint32_t thr_bytes = s.thr ? static_cast<uint32_t>(p.nt * kThrStride * 4) : 0u;
+        const uint32_t tap_bytes = round_up(static_cast<uint32_t>((p.taps + 3) * p.nt * 4), 16);
+        bool placed = false;
+        for (int as : {3, 2}) {
+            for (int rs : {3, 2}) {
+                uint32_t off = 0;
+                const uint32_t off_b = off;
+                off = round_up(off + b_bytes, 128);
+                const uint32_t off_a = off;
+                off = round_up(off + as * stage_bytes, 128);
+                const uint32_t off_raw = off;
+                off = round_up(off + rs * raw_bytes, 128);
+                const uint32_t off_rec = off;
+                off += rec_bytes;
+                const uint32_t off_thr = off;
+                off += thr_bytes;
+                const uint32_t off_tap = off;
+                off += tap_bytes;
+                const uint32_t off_bar = round_up(off, 16);
+                const uint32_t total = off_bar + kBarBytes;
+                // descriptor start addresses are 14-bit fields of 16-byte units (256 KB)
+                if (total > static_cast<uint32_t>(win::kSmemLimit)) continue;
+                p.a_stages = as;
+                p.raw_stages = rs;
+                p.off_b = off_b;
+                p.off_a = off_a;
+                p.off_raw = off_raw;
+                p.off_rec = off_rec;
+                p.off_thr = off_thr;
+                p.off_tap = off_tap;
+                p.off_bar = off_bar;
+                p.smem_bytes = total;
+                placed = true;
+                break;
+            }
+            if (placed) break;
+        }
+        if (!placed) continue;
+        p.s = S;
+        p.sp = sp;
+        p.wh = wh;
+        p.p_alloc = static_cast<int>(p_alloc);
+        p.tiles_x = tiles_x;
+        p.tiles_y = (s.oh + win::kRows - 1) / win::kRows;
+        p.tiles_per_img = p.tiles_x * p.tiles_y;
+        p.total_tiles = static_cast<long long>(s.n) * p.tiles_per_img;
+        if (p.total_tiles >= (1ll << 31)) return p;
+        p.full_rows = full_rows;
+        p.raw_row_bytes = raw_row_bytes;
+        p.raw_bytes = raw_bytes;
+        p.b_bytes = b_bytes;
+        p.chunk_stride = chunk_stride;
+        p.stage_bytes = stage_bytes;
+        // prepared workspace: the packed filters, bias, kappa, lambda and shifts
+        const size_t wbytes = static_cast<size_t>(s.m) * p.taps * static_cast<size_t>(cb);
+        p.off_pw = 0;
+        p.off_pbias = round_up_sz(wbytes, 256);
+        p.off_pkappa = round_up_sz(p.off_pbias + 4 * static_cast<size_t>(s.m), 256);
+        p.off_plambda = round_up_sz(p.off_pkappa + 2 * static_cast<size_t>(s.m), 256);
+        p.off_pshifts = round_up_sz(p.off_plambda + 4 * static_cast<size_t>(s.m), 256);
+        p.off_pthr = round_up_sz(p.off_pshifts + static_cast<size_t>(s.m), 256);
+        p.param_bytes = p.off_pthr;
+        p.ok = true;
+        return p;
+    }
+    return p;
+}
+
+cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, cudaStream_t st)
+{
+    if (s.n == 0) return cudaSuccess;
+    win::WinArgs a{};
+    a.x = p.x;
+    a.y = p.y;
+    a.w = p.w;
+    a.bias = p.bias;
+    a.kappa = p.kappa;
+    a.lambda = p.lambda;
+    a.shifts = p.shifts;
+    a.thr = s.thr ? p.thresholds : nullptr;
+    a.shift = p.shift;
+    a.n = s.n; a.h = s.h; a.w_ = s.w; a.c = s.c; a.m = s.m; a.kh = s.kh; a.kw = s.kw;
+    a.ph = s.ph; a.pw = s.pw; a.oh = s.oh; a.ow = s.ow;
+    a.c_pad = plan.c_pad;
+    a.groups = plan.groups;
+    a.taps = plan.taps;
+    a.ksteps = plan.ksteps;
+    a.s = plan.s;
+    a.sp = plan.sp;
+    a.wh = plan.wh;
+    a.npos = plan.wh * plan.sp;
+    a.cb = s.c * s.bits / 8;
+    a.full_rows = plan.full_rows;
+    a.tiles_x = plan.tiles_x;
+    a.tiles_per_img = plan.tiles_per_img;
+    a.total_tiles = static_cast<int>(plan.total_tiles);
+    a.fd_tpi = make_fastdiv(static_cast<uint32_t>(plan.tiles_per_img));
+    a.fd_tx = make_fastdiv(static_cast<uint32_t>(plan.tiles_x));
+    a.fd_sp = make_fastdiv(static_cast<uint32_t>(plan.sp));
+    a.raw_stages = plan.raw_stages;
+    a.a_stages = plan.a_stages;
+    a.nch_max = plan.nch_max;
+    a.raw_row_bytes = plan.raw_row_bytes;
+    a.raw_bytes = plan.raw_bytes;
+    a.chunk_stride = plan.chunk_stride;
+    a.stage_bytes = plan.stage_bytes;
+    a.off_b = plan.off_b;
+    a.off_a = plan.off_a;
+    a.off_raw = plan.off_raw;
+    a.off_rec = plan.off_rec;
+    a.off_thr = plan.off_thr;
+    a.off_tap = plan.off_tap;
+    a.off_bar = plan.off_bar;
+    a.pool = s.pool;
+    a.pool_oh = s.oh / 2;
+    a.pool_ow = s.ow / 2;
+    for (int i = 0; i < s.kh; ++i)
+        for (int j = 0; j < s.kw; ++j) a.tap_a16[i * s.kw + j] = static_cast<uint32_t>(i * plan.sp + j);
+    a.status = device_status_ptr();
+    if (!a.status) return cudaErrorInvalidSymbol;
+    const long long sms = device_sm_count();
+    const int grid = static_cast<int>(std::min<long long>(plan.total_tiles, sms));
+    switch (s.bits) {
+        case 8: return launch_win_bits<8>(a, plan.nt, grid, plan.smem_bytes, st);
+        case 4: return launch_win_bits<4>(a, plan.nt, grid, plan.smem_bytes, st);
+        default: return launch_win_bits<2>(a, plan.nt, grid, plan.smem_bytes, st);
+    }
+}
+
+cudaError_t prepare_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
+                             cudaStream_t st)
+{
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    const size_t wbytes = static_cast<size_t>(s.m) * plan.taps * (static_cast<size_t>(s.c) * s.bits / 8);
+    cudaError_t e = cudaMemcpyAsync(ws + plan.off_pw, p.w, wbytes, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess)
+        e = p.bias ? cudaMemcpyAsync(ws + plan.off_pbias, p.bias, 4 * static_cast<size_t>(s.m),
+                                     cudaMemcpyDeviceToDevice, st)
+                   : cudaMemsetAsync(ws + plan.off_pbias, 0, 4 * static_cast<size_t>(s.m), st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(ws + plan.off_pkappa, p.kappa, 2 * static_cast<size_t>(s.m), cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(ws + plan.off_plambda, p.lambda, 4 * static_cast<size_t>(s.m), cudaMemcpyDeviceToDevice,
+                            st);
+    if (e == cudaSuccess)
+        e = p.shifts ? cudaMemcpyAsync(ws + plan.off_pshifts, p.shifts, static_cast<size_t>(s.m),
+                                       cudaMemcpyDeviceToDevice, st)
+                     : cudaMemsetAsync(ws + plan.off_pshifts, p.shift, static_cast<size_t>(s.m), st);
+    return e;
+}
+
+ConvParams win_prepared_params(const WinPlan &plan, const void *workspace)
+{
+    const uint8_t *ws = static_cast<const uint8_t *>(workspace);
+    ConvParams p{};
+    p.w = ws + plan.off_pw;
+    p.bias = reinterpret_cast<const int32_t *>(ws + plan.off_pbias);
+    p.kappa = reinterpret_cast<const int16_t *>(ws + plan.off_pkappa);
+    p.lambda = reinterpret_cast<const int32_t *>(ws + plan.off_plambda);
+    p.shifts = ws + plan.off_pshifts;
+    p.shift = 0;
+    p.thresholds = nullptr;
+    return p;
+}
+
+}  // namespace qnn

@@ -1,0 +1,54 @@
+// Instantiations of the window kernel for one bit width (QNN_WIN_BITS), by
+// output-channel tile and fused pool.  Included once by each conv_win_q*.cu.
+#pragma once
+
+#include <mutex>
+
+#include "conv_win.cuh"
+
+#ifndef QNN_WIN_BITS
+#error "define QNN_WIN_BITS (8, 4 or 2) before including conv_win_inst.cuh"
+#endif
+
+namespace qnn {
+namespace {
+
+template <int BITS, int NT, bool POOL>
+cudaError_t launch_one(const win::WinArgs &a, int grid, uint32_t smem, cudaStream_t st)
+{
+    // the opt-in shared-memory limit is raised once per device, outside any stream capture
+    static std::mutex mu;
+    static bool raised[64] = {};
+    auto kern = win::conv_win_kernel<BITS, NT, POOL>;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+        if (!raised[dev]) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, win::kSmemLimit);
+            if (e != cudaSuccess) return e;
+            raised[dev] = true;
+        }
+    }
+    kern<<<grid, win::kThreads, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+template <>
+cudaError_t launch_win_bits<QNN_WIN_BITS>(const win::WinArgs &a, int nt, int grid, uint32_t smem, cudaStream_t st)
+{
+    constexpr int B = QNN_WIN_BITS;
+    switch (nt) {
+        case 32: return a.pool ? launch_one<B, 32, true>(a, grid, smem, st) : launch_one<B, 32, false>(a, grid, smem, st);
+        case 64: return a.pool ? launch_one<B, 64, true>(a, grid, smem, st) : launch_one<B, 64, false>(a, grid, smem, st);
+        case 128:
+            return a.pool ? launch_one<B, 128, true>(a, grid, smem, st) : launch_one<B, 128, false>(a, grid, smem, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace qnn

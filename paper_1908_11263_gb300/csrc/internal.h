@@ -73,6 +73,45 @@ cudaError_t launch_conv_tc_prep(const TcPlan &plan, const ConvShape &s, const Co
 cudaError_t launch_conv_tc_run(const TcPlan &plan, const ConvShape &s, const uint8_t *x, uint8_t *y,
                                const void *workspace, cudaStream_t st, bool after_prep);
 
+// ---- tensor-core window kernel (stride 1, one launch per layer) -- conv_win*.cu
+// Tiles of S strips (16 output rows x 8 columns each) staged as one padded
+// window; filters re-laid out and per-channel constants derived in shared
+// memory by the kernel itself; exact-chunk count derived from the filters.
+struct WinPlan {
+    bool ok;
+    int nt;               // MMA N: all output channels, rounded up to 32, 64 or 128
+    int fp8;              // e4m3 staging, kind::f8f6f4 (INT-4/INT-2), else fp16, kind::f16 (INT-8)
+    int kch;              // channels per 16-byte K-chunk: 8 (fp16) or 16 (e4m3)
+    int c_pad;            // channels per tap rounded up to two K-chunks
+    int groups;           // K-chunks per tap (c_pad / kch)
+    int taps;             // kh * kw
+    int ksteps;           // MMAs per tap (groups / 2)
+    int s;                // strips per tile (1 or 2)
+    int sp, wh;           // window width and height in pixels
+    int p_alloc;          // staged positions per K-chunk plane
+    int tiles_x, tiles_y, tiles_per_img;
+    long long total_tiles;
+    int full_rows;        // a window spans whole image rows: one bulk copy per tile
+    int nch_max;          // exact fp32 chunks the worst-case filters would need
+    int raw_stages, a_stages;
+    uint32_t raw_row_bytes, raw_bytes, b_bytes, chunk_stride, stage_bytes;
+    uint32_t off_b, off_a, off_raw, off_rec, off_thr, off_tap, off_bar, smem_bytes;
+    size_t param_bytes;   // qconv_hwc_prepare workspace: copies of the filters and constants
+    size_t off_pw, off_pbias, off_pkappa, off_plambda, off_pshifts, off_pthr;  // within it
+};
+
+WinPlan plan_conv_win(const ConvShape &s);
+// One launch: the window kernel reads the caller's filters and constants (p.w,
+// p.bias, ...), or copies of them that qconv_hwc_prepare placed in a workspace.
+cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, cudaStream_t st);
+// qconv_hwc_prepare for the window kernel: copies filters and constants into
+// the workspace (device-to-device copies on `st`), laid out as the plan says.
+cudaError_t prepare_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
+                             cudaStream_t st);
+// ConvParams pointing at the copies in a prepared workspace (bias and per-channel
+// shifts always present there: zeros and the scalar shift when the caller gave none).
+ConvParams win_prepared_params(const WinPlan &plan, const void *workspace);
+
 // ---- max-pool, fully connected, packing
 cudaError_t launch_maxpool(int n, int h, int w, int c, int k, int s, int bits, const uint8_t *x, uint8_t *y,
                            cudaStream_t st);

@@ -22,12 +22,12 @@ from . import build as _build
 QNN_OK, QNN_EINVAL, QNN_EUNSUPPORTED, QNN_EALIGN, QNN_ECUDA, QNN_ETIMEOUT, QNN_EWORKSPACE = range(7)
 QNN_ESCRATCH = 7
 NOALLOC_SCRATCH_BYTES = 2 << 20  # QNN_NOALLOC_SCRATCH_BYTES
-ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE = 0, 1, 2
+ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE, ALGO_TC_WINDOW, ALGO_TC_GENERAL = 0, 1, 2, 3, 4
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
             "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
             "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary", "qconv_hwc_pool2",
-            "qconv_hwc_mma_operand_bits")
+            "qconv_hwc_mma_operand_bits", "qconv_hwc_tc_kernel")
 
 
 class QnnError(RuntimeError):
@@ -83,6 +83,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_algo.restype = I32
         lib.qconv_hwc_mma_operand_bits.argtypes = [DP]
         lib.qconv_hwc_mma_operand_bits.restype = I32
+        lib.qconv_hwc_tc_kernel.argtypes = [DP]
+        lib.qconv_hwc_tc_kernel.restype = I32
         lib.qlinear.argtypes = [I32, I32, I32, P, P, P, P, P]
         lib.qlinear.restype = I32
         lib.qmaxpool.argtypes = [I32] * 7 + [P, P, P]
@@ -154,6 +156,15 @@ def conv_algo(desc: ConvDesc) -> int:
     return r
 
 
+def tc_kernel(desc: ConvDesc) -> int:
+    """The tensor-core kernel qconv_hwc() runs for this descriptor: ALGO_TC_WINDOW or
+    ALGO_TC_GENERAL (0 for the CUDA-core kernel)."""
+    r = load().qconv_hwc_tc_kernel(ctypes.byref(desc))
+    if r < 0:
+        raise QnnError(-r, "qconv_hwc_tc_kernel")
+    return r
+
+
 def mma_operand_bits(desc: ConvDesc) -> int:
     """Operand width of the tensor-core MMAs for this descriptor: 16 (fp16, kind::f16),
     8 (e4m3, kind::f8f6f4) or 0 (CUDA-core kernel)."""
@@ -212,8 +223,8 @@ def conv_hwc(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, strid
     return out
 
 
-def conv_hwc_pool2(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, pad=0, out=None, workspace=None,
-                   stream=None):
+def conv_hwc_pool2(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8, pad=0, algo=ALGO_AUTO, out=None,
+                   workspace=None, stream=None):
     """Quantized HWC convolution (stride 1) with fused compression and 2x2 stride-2 max-pooling
     (qconv_hwc_pool2); returns uint8 [n, oh // 2, ow // 2, m*Q/8]."""
     _dev(x, torch.uint8, "x")
@@ -229,7 +240,7 @@ def conv_hwc_pool2(x, w, kappa, lam, *, bias=None, shifts=None, shift=0, bits=8,
     m, kh, kw, cb2 = w.shape
     if cb != cb2:
         raise ValueError("x and w disagree on the channel count")
-    desc = conv_desc(n, h, wd, cb * per, m, kh, kw, 1, pad, bits, shift, ALGO_AUTO)
+    desc = conv_desc(n, h, wd, cb * per, m, kh, kw, 1, pad, bits, shift, algo)
     oh = h + 2 * desc.pad_h - kh + 1
     ow = wd + 2 * desc.pad_w - kw + 1
     if out is None:
@@ -347,13 +358,13 @@ class PreparedConv:
     (qconv_hwc_prepare); calling it runs only the convolution (qconv_hwc_run)."""
 
     def __init__(self, w, kappa, lam, *, n, h, wd, bias=None, shifts=None, shift=0, bits=8, stride=1, pad=0,
-                 stream=None):
+                 algo=ALGO_TENSORCORE, stream=None):
         _dev(w, (torch.int8, torch.uint8), "w")
         _dev(kappa, torch.int16, "kappa")
         _dev(lam, torch.int32, "lambda")
         per = 8 // bits
         m, kh, kw, cb = w.shape
-        self.desc = conv_desc(n, h, wd, cb * per, m, kh, kw, stride, pad, bits, shift, ALGO_TENSORCORE)
+        self.desc = conv_desc(n, h, wd, cb * per, m, kh, kw, stride, pad, bits, shift, algo)
         self.oh = (h + 2 * self.desc.pad_h - kh) // self.desc.stride_h + 1
         self.ow = (wd + 2 * self.desc.pad_w - kw) // self.desc.stride_w + 1
         self.out_shape = (n, self.oh, self.ow, m // per)

@@ -80,6 +80,24 @@ def conv_oracle(x, w, bias, kappa, lam, shifts, shift, bits, stride, pad):
     return oracle.conv_hwc(xp, wp, shape, bias, kappa, lam, shifts=shifts, shift=shift, nthreads=THREADS)
 
 
+def tc_algos(n, h, w, c, m, kh, kw, stride=(1, 1), pad=(0, 0), bits=8):
+    """The tensor-core kernels that can run this layer, each as the algorithm value that forces it
+    (the window kernel, the general kernel)."""
+    out = []
+    for algo in (qnn.ALGO_TC_WINDOW, qnn.ALGO_TC_GENERAL):
+        try:
+            qnn.conv_algo(qnn.conv_desc(n, h, w, c, m, kh, kw, stride, pad, bits, 0, algo))
+            out.append(algo)
+        except qnn.QnnError:
+            pass
+    return out
+
+
+def all_algos(n, h, w, c, m, kh, kw, stride=(1, 1), pad=(0, 0), bits=8):
+    """Every kernel that can run this layer: the tensor-core kernels and the CUDA-core one."""
+    return tc_algos(n, h, w, c, m, kh, kw, stride, pad, bits) + [qnn.ALGO_DIRECT]
+
+
 def first_mismatch(got, want):
     bad = np.nonzero(got != want)[0]
     if bad.size == 0:

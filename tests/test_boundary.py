@@ -81,6 +81,11 @@ def conv_status(lib, d, x=FAKE, w=FAKE, bias=FAKE, kappa=FAKE, lam=FAKE, shifts=
     (dict(bits=4, c=33), qnn.QNN_EUNSUPPORTED), (dict(bits=2, m=62), qnn.QNN_EUNSUPPORTED),
     (dict(c=40000, kh=1, kw=1, pad=(0, 0)), qnn.QNN_EUNSUPPORTED),  # accumulator bound
     (dict(algo=7), qnn.QNN_EINVAL), (dict(stride=(2, 2), algo=qnn.ALGO_TENSORCORE), qnn.QNN_EUNSUPPORTED),
+    # the window kernel: stride 1, whole 8-channel chunks at INT-8, at most 128 output channels
+    (dict(stride=(2, 2), algo=qnn.ALGO_TC_WINDOW), qnn.QNN_EUNSUPPORTED),
+    (dict(c=12, algo=qnn.ALGO_TC_WINDOW), qnn.QNN_EUNSUPPORTED),
+    (dict(m=136, algo=qnn.ALGO_TC_WINDOW), qnn.QNN_EUNSUPPORTED),
+    (dict(stride=(2, 2), algo=qnn.ALGO_TC_GENERAL), qnn.QNN_EUNSUPPORTED),
 ])
 def test_conv_descriptor_validation(lib, kw, code):
     assert conv_status(lib, desc(**kw)) == code
@@ -98,9 +103,12 @@ def test_conv_pointer_and_alignment_validation(lib):
     assert conv_status(lib, d, w=FAKE + 4) == qnn.QNN_EALIGN
     assert conv_status(lib, d, bias=FAKE + 2) == qnn.QNN_EALIGN
     assert conv_status(lib, d, kappa=FAKE + 1) == qnn.QNN_EALIGN
-    assert conv_status(lib, d, ws=0) == qnn.QNN_EWORKSPACE
-    assert conv_status(lib, d, wsb=16) == qnn.QNN_EWORKSPACE
-    assert conv_status(lib, d, ws=FAKE + 16) == qnn.QNN_EWORKSPACE
+    # the general tensor-core kernel needs its workspace (the window kernel, which this layer
+    # takes by default, reads the filters in place and needs none)
+    g = desc(algo=qnn.ALGO_TC_GENERAL)
+    assert conv_status(lib, g, ws=0) == qnn.QNN_EWORKSPACE
+    assert conv_status(lib, g, wsb=16) == qnn.QNN_EWORKSPACE
+    assert conv_status(lib, g, ws=FAKE + 16) == qnn.QNN_EWORKSPACE
     bad = desc()
     bad.struct_size = 8
     assert conv_status(lib, bad) == qnn.QNN_EINVAL
@@ -112,8 +120,8 @@ def test_algo_selection_and_workspace(lib):
     assert qnn.conv_algo(desc(stride=(2, 2))) == qnn.ALGO_DIRECT
     assert qnn.conv_algo(desc(algo=qnn.ALGO_DIRECT)) == qnn.ALGO_DIRECT
     assert qnn.workspace_size(desc(algo=qnn.ALGO_DIRECT)) == 0
-    ws = qnn.workspace_size(desc())
-    # fp16 filters (64 x 3*3*32) plus 16 bytes of constants per channel
+    ws = qnn.workspace_size(desc(algo=qnn.ALGO_TC_GENERAL))
+    # general kernel: fp16 filters (64 x 3*3*32) plus 16 bytes of constants per channel
     assert ws >= 64 * 288 * 2 + 64 * 16
     for bits in (4, 2):
         assert qnn.conv_algo(desc(bits=bits)) == qnn.ALGO_TENSORCORE
@@ -122,14 +130,15 @@ def test_algo_selection_and_workspace(lib):
 
 
 def test_subbyte_layers_with_c_multiple_of_32_plan_e4m3_filters(lib):
-    """INT-4/INT-2 layers whose C is a multiple of 32 stage e4m3 bytes (one byte per filter
-    element in the workspace); INT-8 and C = 16 keep fp16 (two bytes). The workspace is the
-    filters plus 96 bytes of per-channel constants and thresholds."""
+    """The general kernel: INT-4/INT-2 layers whose C is a multiple of 32 stage e4m3 bytes (one
+    byte per filter element in the workspace); INT-8 and C = 16 keep fp16 (two bytes). Its
+    workspace is the filters plus 96 bytes of per-channel constants and thresholds."""
     consts = 64 * (32 + 64)
-    assert qnn.workspace_size(desc()) == 64 * 3 * 3 * 32 * 2 + consts
+    g = qnn.ALGO_TC_GENERAL
+    assert qnn.workspace_size(desc(algo=g)) == 64 * 3 * 3 * 32 * 2 + consts
     for bits in (4, 2):
-        assert qnn.workspace_size(desc(bits=bits)) == 64 * 3 * 3 * 32 * 1 + consts
-        d16 = qnn.conv_desc(1, 8, 8, 16, 64, 3, 3, 1, 1, bits, 10)
+        assert qnn.workspace_size(desc(bits=bits, algo=g)) == 64 * 3 * 3 * 32 * 1 + consts
+        d16 = qnn.conv_desc(1, 8, 8, 16, 64, 3, 3, 1, 1, bits, 10, g)
         assert qnn.workspace_size(d16) == 64 * 3 * 3 * 16 * 2 + consts
         # the operand-format query agrees: e4m3 (8 bits) with C = 32, fp16 with C = 16
         assert qnn.mma_operand_bits(desc(bits=bits)) == 8
@@ -138,6 +147,25 @@ def test_subbyte_layers_with_c_multiple_of_32_plan_e4m3_filters(lib):
     assert qnn.mma_operand_bits(desc(stride=(2, 2))) == 0
     with pytest.raises(qnn.QnnError):
         qnn.mma_operand_bits(desc(bits=5))
+
+
+def test_window_kernel_selection_and_prepared_workspace(lib):
+    """Tensor-core requests take the window kernel where its plan fits (the benchmark layer at
+    every Q, the CIFAR-shaped conv2 / conv3) and the general kernel elsewhere (C = 3, more than
+    128 output channels).  The window kernel's prepared workspace holds copies of the packed
+    filters, bias, kappa, lambda and shifts, each 256-byte aligned."""
+    for bits in (8, 4, 2):
+        assert qnn.tc_kernel(desc(bits=bits)) == qnn.ALGO_TC_WINDOW
+    assert qnn.tc_kernel(qnn.conv_desc(1024, 16, 16, 32, 32, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_WINDOW
+    assert qnn.tc_kernel(qnn.conv_desc(1024, 8, 8, 32, 64, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_WINDOW
+    assert qnn.tc_kernel(qnn.conv_desc(1024, 32, 32, 3, 32, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_GENERAL
+    assert qnn.tc_kernel(qnn.conv_desc(64, 14, 14, 256, 512, 1, 1, 1, 0, 8, 10)) == qnn.ALGO_TC_GENERAL
+    assert qnn.tc_kernel(desc(algo=qnn.ALGO_TC_GENERAL)) == qnn.ALGO_TC_GENERAL
+    assert qnn.tc_kernel(desc(stride=(2, 2))) == 0
+    # 64 x 3x3x32 bytes of filters, then int32 bias, int16 kappa, int32 lambda, uint8 shifts
+    r = lambda v: (v + 255) // 256 * 256  # noqa: E731
+    wbytes = 64 * 9 * 32
+    assert qnn.workspace_size(desc()) == r(r(r(r(wbytes) + 4 * 64) + 2 * 64) + 4 * 64) + 256
 
 
 def test_other_entry_points_validate(lib):

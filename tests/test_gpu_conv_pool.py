@@ -9,7 +9,7 @@ import torch
 import oracle
 from paper_1908_11263_gb300 import build as qbuild
 from paper_1908_11263_gb300 import qnn
-from gpu_util import THREADS, check_guard, first_mismatch, guarded_output, pack_gpu, to_dev
+from gpu_util import THREADS, check_guard, first_mismatch, guarded_output, pack_gpu, tc_algos, to_dev
 
 FAKE = 0x10000  # 16-byte aligned, never dereferenced: validation fails first
 
@@ -38,7 +38,7 @@ def packed_dev(v, bits, shape):
     return t.view(*shape[:-1], shape[-1] // per)
 
 
-def run_fused(x, wt, bias, kappa, lam, shifts, shift, bits, pad):
+def run_fused(x, wt, bias, kappa, lam, shifts, shift, bits, pad, algo=qnn.ALGO_AUTO):
     n, h, w, c = x.shape
     m, k, _, _ = wt.shape
     per = 8 // bits
@@ -49,7 +49,7 @@ def run_fused(x, wt, bias, kappa, lam, shifts, shift, bits, pad):
         wd = wd.view(torch.int8)
     qnn.conv_hwc_pool2(packed_dev(x, bits, x.shape), wd, to_dev(kappa, torch.int16), to_dev(lam, torch.int32),
                        bias=to_dev(bias, torch.int32), shifts=None if shifts is None else to_dev(shifts, torch.uint8),
-                       shift=shift, bits=bits, pad=pad, out=out)
+                       shift=shift, bits=bits, pad=pad, algo=algo, out=out)
     qnn.device_status()
     check_guard(buf)
     return out, wd
@@ -89,9 +89,12 @@ def test_conv_pool2_matches_oracle(shape):
     n, h, w, c, m, k, pad, bits = shape
     case = spread_case(hash(shape) & 0xFFFF, n, h, w, c, m, k, bits, per_channel_shift=(h % 2 == 0))
     want = run_oracle(*case, bits, pad)
-    out, _ = run_fused(*case, bits, pad)
-    got = out.cpu().numpy().reshape(-1)
-    assert first_mismatch(got, want) is None, first_mismatch(got, want)
+    algos = tc_algos(n, h, w, c, m, k, k, (1, 1), (pad, pad), bits)
+    assert algos
+    for algo in algos:
+        out, _ = run_fused(*case, bits, pad, algo)
+        got = out.cpu().numpy().reshape(-1)
+        assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
     assert len(np.unique(want)) > 4, "pooled outputs nearly constant: the check is weak"
 
 
@@ -121,13 +124,15 @@ def test_conv_pool2_cifar_chain_batch1024():
     xo = x.astype(np.uint8).reshape(-1)
     for key, layer, wl, lid in inputs.cifar_layers(n):
         ld = inputs.make_layer(key, layer, wl, lid, x=np.zeros(1))
-        yd = qnn.conv_hwc_pool2(xd, to_dev(ld.w), to_dev(ld.kappa, torch.int16), to_dev(ld.lam, torch.int32),
-                                bias=to_dev(ld.bias, torch.int32), shift=ld.shift, bits=8, pad=layer.pad)
-        qnn.device_status()
         yo = oracle.conv_hwc_pool2(xo, ld.w.reshape(-1).view(np.uint8), layer.shape(), ld.bias, ld.kappa, ld.lam,
                                    shift=ld.shift, nthreads=THREADS)
-        got = yd.cpu().numpy().reshape(-1)
-        assert first_mismatch(got, yo) is None, (key, first_mismatch(got, yo))
+        for algo in tc_algos(n, layer.h, layer.w, layer.c, layer.m, layer.k, layer.k, (1, 1), (layer.pad, layer.pad), 8):
+            yd = qnn.conv_hwc_pool2(xd, to_dev(ld.w), to_dev(ld.kappa, torch.int16), to_dev(ld.lam, torch.int32),
+                                    bias=to_dev(ld.bias, torch.int32), shift=ld.shift, bits=8, pad=layer.pad,
+                                    algo=algo)
+            qnn.device_status()
+            got = yd.cpu().numpy().reshape(-1)
+            assert first_mismatch(got, yo) is None, (key, algo, first_mismatch(got, yo))
         assert len(np.unique(yo)) > 16, f"{key}: pooled outputs nearly constant, the check is weak"
         xd, xo = yd, yo
     wfc, bfc = inputs.cifar_fc()
@@ -158,4 +163,6 @@ def test_conv_pool2_rejects_what_it_cannot_run(lib):
     assert status(qnn.conv_desc(1, 8, 3, 32, 32, 3, 3, 1, 0, 8, 10)) == qnn.QNN_EINVAL
     assert status(ok, x=0) == qnn.QNN_EINVAL
     assert status(ok, y=FAKE + 8) == qnn.QNN_EALIGN
-    assert status(ok, ws=0) == qnn.QNN_EWORKSPACE
+    # the general kernel needs its workspace; the window kernel (this layer's default) reads the
+    # filters in place
+    assert status(qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 1, 1, 8, 10, qnn.ALGO_TC_GENERAL), ws=0) == qnn.QNN_EWORKSPACE

@@ -9,7 +9,7 @@ import torch
 import oracle
 from paper_1908_11263_gb300 import build as qbuild
 from paper_1908_11263_gb300 import qnn
-from gpu_util import check_guard, dev, first_mismatch, guarded_output, pack_gpu, to_dev
+from gpu_util import check_guard, dev, first_mismatch, guarded_output, pack_gpu, tc_algos, to_dev
 
 FAKE = 0x10000
 
@@ -64,7 +64,7 @@ def test_thresholds_match_oracle(bits, shape):
     tau = sorted_thresholds(rng, m, bits, k * k * c)
     want = run_oracle(x, wt, tau, bits, stride, pad)
     assert len(np.unique(want)) > 4
-    algos = [qnn.ALGO_DIRECT] + ([qnn.ALGO_TENSORCORE] if stride == 1 else [])
+    algos = [qnn.ALGO_DIRECT] + (tc_algos(n, h, w, c, m, k, k, (1, 1), (pad, pad), bits) if stride == 1 else [])
     for algo in algos:
         got = run_gpu(x, wt, tau, bits, stride, pad, algo)
         assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
@@ -81,7 +81,7 @@ def test_unsorted_thresholds_count(bits):
     tau = rng.integers(centre - 200, centre + 200, size=(32, top)).astype(np.int32)
     want = run_oracle(x, wt, tau, bits, 1, 1)
     assert len(np.unique(want)) > 4
-    for algo in (qnn.ALGO_DIRECT, qnn.ALGO_TENSORCORE):
+    for algo in [qnn.ALGO_DIRECT] + tc_algos(2, 10, 16, 32, 32, 3, 3, (1, 1), (1, 1), bits):
         got = run_gpu(x, wt, tau, bits, 1, 1, algo)
         assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
 
@@ -104,7 +104,7 @@ def test_affine_thresholds_equal_scaling_and_clip_on_gpu(bits):
     wd_ = pack_gpu(wt, bits).view(m, k, k, c // per)
     ref = qnn.conv_hwc(xd, wd_, to_dev(kappa, torch.int16), to_dev(lam, torch.int32), bias=to_dev(bias, torch.int32),
                        shift=shift, bits=bits, pad=1)
-    for algo in (qnn.ALGO_DIRECT, qnn.ALGO_TENSORCORE):
+    for algo in [qnn.ALGO_DIRECT] + tc_algos(n, h, w, c, m, k, k, (1, 1), (1, 1), bits):
         got = qnn.conv_hwc_thresholds(xd, wd_, to_dev(tau, torch.int32), bits=bits, pad=1, algo=algo)
         assert torch.equal(got, ref), algo
 

@@ -1,0 +1,106 @@
+"""The window tensor-core kernel (one launch per call, filters read in place, exact-chunk
+count derived from the filters) and the prepared path (qconv_hwc_prepare + qconv_hwc_run) of
+both tensor-core kernels, against the oracle bit for bit (Sec. III-B, Eq. 6; Sec. III-A)."""
+import numpy as np
+import pytest
+import torch
+
+from paper_1908_11263_gb300 import qnn
+
+from gpu_util import conv_gpu, conv_oracle, first_mismatch, pack_gpu, tc_algos, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def loaded():
+    qnn.load(build_if_missing=True)
+    torch.cuda.set_device(0)
+
+
+def centred_lambda(x, wt, bits):
+    """kappa = 1, shift = 0 and a per-channel lambda that centres each channel's accumulators
+    in the output range: every output then depends on the accumulator's last bit."""
+    import oracle
+    acc = oracle.conv_acc(x, wt, (1, 1), (1, 1)).reshape(-1, wt.shape[0])
+    half = 1 << (bits - 1)
+    return (half - np.median(acc, axis=0)).astype(np.int32)
+
+
+# (n, h, w, c, m, k): the benchmark layer's shape, C = 64 (K = 576) and a 5x5 window (K = 800)
+SHAPES = [(2, 16, 16, 32, 64, 3), (1, 16, 16, 64, 64, 3), (2, 16, 16, 32, 32, 5)]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: "x".join(map(str, s)))
+@pytest.mark.parametrize("pattern", ["uniform", "extreme", "one_extreme_channel", "alternating"])
+def test_chunk_count_from_filters(shape, pattern):
+    """INT-8 filters whose sum |w| decides how many exact fp32 chunks the window kernel takes:
+    uniform random filters allow fewer chunks than the worst case; filters at -128 throughout
+    (one channel, or all) force the worst case for every channel; alternating extremes keep the
+    true sum small while the chunk bound stays large.  Both tensor-core kernels equal the oracle."""
+    n, h, w, c, m, k = shape
+    rng = np.random.default_rng(sum(shape) * 7 + len(pattern))
+    x = rng.integers(0, 256, size=(n, h, w, c))
+    wt = rng.integers(-128, 128, size=(m, k, k, c))
+    if pattern == "extreme":
+        wt[:] = -128
+        x[:] = rng.integers(0, 2, size=x.shape) * 255  # staged values at both ends
+    elif pattern == "one_extreme_channel":
+        wt[m // 3] = -128
+    elif pattern == "alternating":
+        wt[..., 0::2] = 127
+        wt[..., 1::2] = -128
+    lam = centred_lambda(x, wt, 8)
+    kappa = np.ones(m, np.int16)
+    want = conv_oracle(x, wt, None, kappa, lam, None, 0, 8, (1, 1), (1, 1))
+    if pattern != "extreme":
+        assert len(np.unique(want)) > 32, "outputs nearly constant: the check is weak"
+    algos = tc_algos(n, h, w, c, m, k, k, (1, 1), (1, 1), 8)
+    assert qnn.ALGO_TC_WINDOW in algos
+    for algo in algos:
+        got = conv_gpu(x, wt, None, kappa, lam, None, 0, 8, (1, 1), (1, 1), algo)
+        assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
+
+
+@pytest.mark.parametrize("bits", [8, 4, 2])
+def test_benchmark_layer_takes_the_window_kernel(bits):
+    d = qnn.conv_desc(512, 16, 16, 32, 64, 3, 3, 1, 1, bits, 12)
+    assert qnn.tc_kernel(d) == qnn.ALGO_TC_WINDOW
+    assert qnn.mma_operand_bits(d) == (16 if bits == 8 else 8)
+
+
+@pytest.mark.parametrize("algo", [qnn.ALGO_TC_WINDOW, qnn.ALGO_TC_GENERAL])
+@pytest.mark.parametrize("bits", [8, 4, 2])
+@pytest.mark.parametrize("with_bias_and_shifts", [True, False])
+def test_prepared_path(algo, bits, with_bias_and_shifts):
+    """qconv_hwc_prepare once, then qconv_hwc_run on two different inputs: each equals the
+    oracle.  Without bias and per-channel shifts the prepared workspace must stand in zeros
+    and the scalar shift."""
+    # INT-2 rows of a 20-pixel image are 160 B, but a window of it starts at 8-byte pixels, so
+    # the window kernel needs whole-row windows there: 16 pixels wide
+    n, h, w, c, m, k = 3, 14, 20 if bits != 2 else 16, 32, 48, 3
+    assert algo in tc_algos(n, h, w, c, m, k, k, (1, 1), (1, 1), bits)
+    rng = np.random.default_rng(bits * 11 + algo + int(with_bias_and_shifts))
+    top = (1 << bits) - 1
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, k, k, c))
+    taps = k * k * c
+    bias = (taps * top // 4 + rng.integers(-50, 51, size=m)).astype(np.int32) if with_bias_and_shifts else None
+    kappa = rng.integers(1, 300, size=m).astype(np.int16)
+    shift = {8: 14, 4: 10, 2: 8}[bits]
+    lam = rng.integers(0, (top + 1) << (shift - 1), size=m).astype(np.int32)
+    shifts = rng.integers(shift - 2, shift + 3, size=m).astype(np.uint8) if with_bias_and_shifts else None
+    per = 8 // bits
+    wd = pack_gpu(wt, bits).view(m, k, k, c // per)
+    if bits == 8:
+        wd = wd.view(torch.int8)
+    prep = qnn.PreparedConv(wd, to_dev(kappa, torch.int16), to_dev(lam, torch.int32), n=n, h=h, wd=w,
+                            bias=None if bias is None else to_dev(bias, torch.int32),
+                            shifts=None if shifts is None else to_dev(shifts, torch.uint8), shift=shift, bits=bits,
+                            stride=1, pad=1, algo=algo)
+    for trial in range(2):
+        x = rng.integers(0, top + 1, size=(n, h, w, c))
+        want = conv_oracle(x, wt, bias, kappa, lam, shifts, shift, bits, (1, 1), (1, 1))
+        got = prep(pack_gpu(x, bits).view(n, h, w, c // per)).cpu().numpy().reshape(-1)
+        qnn.device_status()
+        assert first_mismatch(got, want) is None, (trial, first_mismatch(got, want))
+        assert len(np.unique(want)) > 4

@@ -53,3 +53,30 @@ def test_plans_keep_every_access_in_bounds(tmp_path):
     }
     for key, want in expect.items():
         assert plans[key].split(" nt=")[0] == "1 " + want, (key, plans[key])
+
+
+def test_window_plans_keep_every_access_in_bounds(tmp_path):
+    """The same for the window kernel's planner (tests/win_bounds.cpp): shared-memory layout,
+    every bulk copy, converter load and store, MMA operand row and the exact-chunk bound."""
+    lib = qbuild.build()
+    cxx = shutil.which("g++") or shutil.which("c++")
+    if cxx is None:
+        pytest.skip("no host C++ compiler")
+    cuda = _cuda_root()
+    exe = str(tmp_path / "win_bounds")
+    subprocess.run([cxx, "-std=c++17", "-O1", f"-I{os.path.join(cuda, 'include')}", os.path.join(HERE, "win_bounds.cpp"),
+                    "-o", exe, lib, f"-Wl,-rpath,{os.path.dirname(lib)}", f"-L{os.path.join(cuda, 'lib64')}",
+                    "-lcudart"], check=True)
+    out = subprocess.run([exe], capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0 and out.stdout.rstrip().endswith("fails=0"), out.stdout[-4000:]
+    text = out.stdout
+    for word in ("S=1", "S=2", "e4m3", "fp16", "full-rows", "row-segments"):
+        assert f" {word} " in text or f" {word}\n" in text, word
+    plans = {line.split(": ok=")[0]: line.split(": ok=")[1] for line in text.splitlines() if ": ok=" in line}
+    # the benchmark layer at every bit width: whole images (two strips) per tile, one bulk copy each
+    for q, fmt in ((8, "fp16"), (4, "e4m3"), (2, "e4m3")):
+        got = plans[f"512x16x16x32->64 k3x3 p1,1 q{q} pool0"]
+        assert got.startswith(f"1 S=2 {fmt} nt=64") and got.endswith("full-rows"), (q, got)
+    # layers the window kernel leaves to the general kernel: C = 3, more than 128 output channels
+    assert plans["1024x32x32x3->32 k5x5 p2,2 q8 pool0"] == "0"
+    assert plans["64x14x14x256->512 k1x1 p0,0 q8 pool0"] == "0"

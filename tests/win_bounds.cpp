@@ -1,0 +1,199 @@
+// Host-side bounds of the window planner, qnn::plan_conv_win (exported by
+// libqnn).  For each layer shape below, every address the window kernel
+// derives from a plan (restated here from the kernel's addressing rules) is
+// checked against the buffers the plan sizes, for every tile of one image:
+//   - shared memory: filters, staged windows, raw windows, records,
+//     thresholds, tap sums, barriers, in that order, within 227 KB, with the
+//     alignments bulk copies and MMA descriptors need;
+//   - every bulk copy of the loader (size, 16-byte alignment of both ends,
+//     inside its raw stage and inside the input tensor);
+//   - every converter load (inside the bytes the loader copied for that row,
+//     and the global element it stands for is the window pixel's) and store
+//     (inside its stage);
+//   - every A row an MMA reads (inside the staged window, and holding the
+//     input pixel that output pixel and tap need), every B row;
+//   - tensor memory: one slot of accumulators within 512 columns;
+//   - exactness: the planner's worst-case chunk count keeps every chunk within
+//     2^22, and its even tap split has no empty chunk;
+//   - the reciprocal division the kernel uses for tile and window indices.
+// Prints one line per plan and "fails=N"; exits non-zero on any failure.
+#include <algorithm>
+#include <cstdint>
+#include <cstdio>
+
+#include "../paper_1908_11263_gb300/csrc/internal.h"
+
+using namespace qnn;
+
+static int fails = 0;
+#define CHECK(c, ...)                                \
+    do {                                             \
+        if (!(c)) {                                  \
+            ++fails;                                 \
+            std::printf("FAIL %s: ", #c);            \
+            std::printf(__VA_ARGS__);                \
+            std::printf("\n");                       \
+        }                                            \
+    } while (0)
+
+// Constants of the kernel (conv_win.cuh).
+static constexpr int kRows = 16, kCols = 8, kConvThreads = 128, kMaxKP = 5, kMaxStages = 4, kMaxSlots = 4;
+static constexpr long long kSmemLimit = 232448;
+static constexpr long long kBarBytes = (4 * kMaxStages + 2 * kMaxSlots + 2) * 8 + 32;
+
+// The kernel's reciprocal division: floor(n * m / 2^64), m = ceil(2^64 / d).
+static int fdiv(long long n, unsigned d)
+{
+    if (d <= 1) return static_cast<int>(n);
+    const unsigned long long m = (~0ull / d) + 1ull;
+    return static_cast<int>((static_cast<unsigned __int128>(static_cast<unsigned long long>(n)) * m) >> 64);
+}
+
+static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int pw, int bits, int pool)
+{
+    ConvShape s{};
+    s.n = n; s.h = h; s.w = w; s.c = c; s.m = m; s.kh = kh; s.kw = kw; s.sh = 1; s.sw = 1;
+    s.ph = ph; s.pw = pw; s.bits = bits; s.pool = pool; s.thr = 0;
+    s.oh = h + 2 * ph - kh + 1;
+    s.ow = w + 2 * pw - kw + 1;
+    if (pool && (s.oh < 2 || s.ow < 2)) return;  // qconv_hwc_pool2 rejects these before planning
+    const WinPlan p = plan_conv_win(s);
+    std::printf("%dx%dx%dx%d->%d k%dx%d p%d,%d q%d pool%d: ok=%d", n, h, w, c, m, kh, kw, ph, pw, bits, pool, p.ok);
+    if (!p.ok) {
+        std::printf("\n");
+        return;
+    }
+    std::printf(" S=%d %s nt=%d sp=%d wh=%d stages=%d/%d nch_max=%d smem=%u %s\n", p.s, p.fp8 ? "e4m3" : "fp16", p.nt,
+                p.sp, p.wh, p.a_stages, p.raw_stages, p.nch_max, p.smem_bytes, p.full_rows ? "full-rows" : "row-segments");
+    const long long cb = static_cast<long long>(c) * bits / 8;
+    const int kch = p.fp8 ? 16 : 8, gbytes = kch * bits / 8;  // packed bytes of one K-chunk
+    const int load = bits == 8 ? 8 : (bits == 4 ? 8 : 4);                         // bytes one converter load reads
+    CHECK(gbytes == (bits == 8 ? 8 : 16 * bits / 8), "gbytes %d", gbytes);
+    const int npos = p.wh * p.sp;
+    // shared memory layout
+    const long long rec_bytes = 2LL * p.nt * 16 + p.nt * 8 + p.nt / 16;
+    CHECK(p.off_b == 0 && p.off_b + p.b_bytes <= p.off_a, "filters");
+    CHECK(p.off_a % 128 == 0 && p.off_a + static_cast<long long>(p.a_stages) * p.stage_bytes <= p.off_raw, "stages");
+    CHECK(p.off_raw % 128 == 0 && p.off_raw + static_cast<long long>(p.raw_stages) * p.raw_bytes <= p.off_rec, "raw");
+    CHECK(p.off_rec % 16 == 0 && p.off_rec + rec_bytes <= p.off_thr, "records");
+    CHECK(p.off_tap + (p.taps + 3LL) * p.nt * 4 <= p.off_bar && p.off_tap % 4 == 0, "tap sums");
+    CHECK(p.off_bar % 16 == 0 && p.off_bar + kBarBytes <= p.smem_bytes && p.smem_bytes <= kSmemLimit, "barriers");
+    CHECK(p.a_stages >= 2 && p.a_stages <= kMaxStages && p.raw_stages >= 2 && p.raw_stages <= kMaxStages, "rings");
+    CHECK(p.raw_bytes % 16 == 0 && p.stage_bytes % 16 == 0 && p.chunk_stride % 16 == 0, "16-byte units");
+    CHECK(p.chunk_stride >= static_cast<unsigned>(npos) * 16 && p.stage_bytes == p.chunk_stride * p.groups, "planes");
+    // MMA descriptors: 14-bit fields of 16-byte units
+    CHECK(p.smem_bytes < (1u << 18) && p.chunk_stride < (1u << 18) && p.sp * 16 < (1 << 18), "descriptor fields");
+    CHECK(p.groups % 2 == 0 && p.ksteps * 2 == p.groups && p.groups <= 8, "k-steps");
+    // converter positions
+    CHECK(npos <= kMaxKP * kConvThreads, "npos %d", npos);
+    // tensor memory and exactness
+    CHECK(p.s * p.nch_max * p.nt <= 512, "tmem");
+    const long long max_prod = p.fp8 ? (bits == 4 ? 15 * 8 : 3 * 2) : 128 * 128;
+    {
+        const int ct = (p.taps + p.nch_max - 1) / p.nch_max;
+        CHECK(static_cast<long long>(ct) * p.c_pad * max_prod <= (1LL << 22), "worst-case chunk");
+        CHECK((p.nch_max - 1) * ct < p.taps, "empty chunk");
+    }
+    CHECK(256 % p.nt == 0 && p.nt >= m, "prep channel per thread");
+    // the filter-prep loads: the last K-chunk of the last channel inside the packed filters
+    CHECK((static_cast<long long>(m - 1) * p.taps + p.taps - 1) * cb + (c * bits / 8 / gbytes - 1) * gbytes + gbytes <=
+              static_cast<long long>(m) * p.taps * cb,
+          "prep loads");
+    CHECK(p.taps * p.groups * p.nt * 16LL == p.b_bytes, "B size");
+    // division used for window positions
+    for (int pos = 0; pos < kMaxKP * kConvThreads; ++pos) CHECK(fdiv(pos, p.sp) == pos / p.sp, "fdiv sp %d", pos);
+    // every tile of the first and the last image
+    const long long x_bytes = static_cast<long long>(n) * h * w * cb;
+    for (int img : {0, n - 1}) {
+        for (int ti = 0; ti < p.tiles_per_img; ++ti) {
+            const long long t = static_cast<long long>(img) * p.tiles_per_img + ti;
+            const int gi = fdiv(t, p.tiles_per_img);
+            CHECK(gi == img, "fdiv tile");
+            const int ty = fdiv(ti, p.tiles_x), tx = ti - ty * p.tiles_x;
+            const int oy0 = ty * kRows, ox0 = tx * kCols * p.s, iy0 = oy0 - ph, ix0 = ox0 - pw;
+            const int r0 = std::min(p.wh, std::max(0, -iy0)), r1 = std::max(r0, std::min(p.wh, h - iy0));
+            const int c0 = std::min(p.sp, std::max(0, -ix0)), c1 = std::max(c0, std::min(p.sp, w - ix0));
+            // loader
+            const long long seg = p.full_rows ? static_cast<long long>(w) * cb : (c1 - c0) * cb;
+            CHECK(static_cast<long long>(r1 - r0) * p.raw_row_bytes <= p.raw_bytes, "raw stage rows");
+            CHECK(seg <= p.raw_row_bytes && seg % 16 == 0 && p.raw_row_bytes % 16 == 0, "copy size");
+            for (int r = r0; r < r1; ++r) {
+                const long long src =
+                    ((static_cast<long long>(img) * h + iy0 + r) * w + (p.full_rows ? 0 : ix0 + c0)) * cb;
+                CHECK(src >= 0 && src + seg <= x_bytes && src % 16 == 0, "copy source row %d", r);
+                CHECK(iy0 + r >= 0 && iy0 + r < h, "copied row inside the image");
+            }
+            if (p.full_rows) CHECK(ix0 + c0 == 0 && ix0 + c1 == w, "whole rows");
+            // converter
+            const int base_col = p.full_rows ? ix0 : -c0;
+            for (int tid = 0; tid < kConvThreads; ++tid)
+                for (int k = 0; k < kMaxKP; ++k) {
+                    const int pos = tid + 128 * k;
+                    if (pos >= npos) continue;
+                    const int r = fdiv(pos, p.sp), px = pos - r * p.sp;
+                    const bool ok = r >= r0 && r < r1 && px >= c0 && px < c1;
+                    const bool inside = iy0 + r >= 0 && iy0 + r < h && ix0 + px >= 0 && ix0 + px < w;
+                    CHECK(ok == inside, "staged pixel inside the image");
+                    for (int gq = 0; gq < p.groups; ++gq) {
+                        CHECK(static_cast<long long>(gq) * p.chunk_stride + pos * 16LL + 16 <= p.stage_bytes, "store");
+                        if (!ok || gq >= c * bits / 8 / gbytes) continue;
+                        const long long src = static_cast<long long>(r - r0) * p.raw_row_bytes + (px + base_col) * cb +
+                                              static_cast<long long>(gq) * gbytes;
+                        CHECK(src >= 0 && src + load <= static_cast<long long>(r1 - r0) * p.raw_row_bytes, "raw load");
+                        // byte q of copied row r stands for global byte row_start + q
+                        const long long row_start =
+                            ((static_cast<long long>(img) * h + iy0 + r) * w + (p.full_rows ? 0 : ix0 + c0)) * cb;
+                        const long long q = src - static_cast<long long>(r - r0) * p.raw_row_bytes;
+                        CHECK(q + load <= seg, "inside the copied span");
+                        const long long want = ((static_cast<long long>(img) * h + iy0 + r) * w + ix0 + px) * cb +
+                                               static_cast<long long>(gq) * gbytes;
+                        CHECK(row_start + q == want, "the pixel's own channels");
+                        CHECK(src % load == 0, "load alignment");
+                    }
+                }
+            // MMA A rows and B rows
+            for (int sj = 0; sj < p.s; ++sj)
+                for (int i = 0; i < kh; ++i)
+                    for (int j = 0; j < kw; ++j)
+                        for (int g = 0; g < kRows; ++g)
+                            for (int col = 0; col < kCols; ++col) {
+                                const int pos = i * p.sp + j + sj * kCols + g * p.sp + col;
+                                CHECK(pos >= 0 && pos < npos, "A row");
+                                const int r = pos / p.sp, px = pos % p.sp;
+                                const int oy = oy0 + g, ox = ox0 + sj * kCols + col;
+                                if (oy < s.oh && ox < s.ow)
+                                    CHECK(iy0 + r == oy - ph + i && ix0 + px == ox - pw + j, "A row pixel");
+                            }
+            for (int tap = 0; tap < p.taps; ++tap)
+                for (int kk = 0; kk < p.ksteps; ++kk)
+                    CHECK((static_cast<long long>(tap) * p.groups + 2 * kk + 2) * p.nt * 16 <= p.b_bytes, "B rows");
+        }
+    }
+}
+
+int main()
+{
+    // n, h, w, c, m, kh, kw, ph, pw, bits: the parity tests' shapes and the workloads'
+    static const int shapes[][10] = {
+        {2, 16, 16, 32, 64, 3, 3, 1, 1, 8},     {1, 16, 16, 32, 64, 3, 3, 1, 1, 4},   {1, 16, 16, 32, 64, 3, 3, 1, 1, 2},
+        {3, 10, 10, 16, 16, 3, 3, 1, 1, 8},     {2, 14, 14, 64, 48, 3, 3, 1, 1, 8},   {1, 15, 20, 24, 40, 3, 3, 1, 1, 8},
+        {1, 12, 12, 3, 32, 5, 5, 2, 2, 8},      {2, 8, 8, 32, 64, 5, 5, 2, 2, 8},     {1, 7, 7, 128, 136, 3, 3, 1, 1, 8},
+        {1, 6, 6, 256, 256, 3, 3, 1, 1, 8},     {1, 5, 9, 32, 16, 3, 2, 0, 1, 8},     {1, 11, 13, 16, 32, 2, 4, 1, 2, 8},
+        {1, 1, 40, 16, 16, 1, 3, 0, 1, 8},      {2, 13, 13, 32, 24, 3, 3, 0, 0, 4},   {1, 10, 12, 48, 32, 5, 5, 2, 2, 4},
+        {2, 9, 9, 64, 64, 3, 3, 1, 1, 2},       {1, 9, 7, 8, 12, 3, 3, 1, 1, 2},      {1, 16, 16, 12, 16, 3, 3, 1, 1, 4},
+        {512, 16, 16, 32, 64, 3, 3, 1, 1, 8},   {512, 16, 16, 32, 64, 3, 3, 1, 1, 4}, {512, 16, 16, 32, 64, 3, 3, 1, 1, 2},
+        {1024, 32, 32, 3, 32, 5, 5, 2, 2, 8},   {1024, 16, 16, 32, 32, 5, 5, 2, 2, 8}, {1024, 8, 8, 32, 64, 5, 5, 2, 2, 8},
+        {64, 56, 56, 64, 64, 3, 3, 1, 1, 8},    {64, 28, 28, 128, 128, 3, 3, 1, 1, 8}, {64, 14, 14, 256, 256, 3, 3, 1, 1, 8},
+        {64, 14, 14, 256, 512, 1, 1, 0, 0, 8},  {1, 4, 32, 256, 16, 1, 1, 0, 0, 8},   {1, 6, 6, 256, 32, 3, 3, 1, 1, 4},
+        {1, 8, 8, 32, 32, 3, 3, 1, 1, 8},       {2, 30, 16, 32, 64, 3, 3, 1, 1, 8},   {1, 16, 24, 32, 48, 5, 5, 2, 2, 8},
+        {1, 47, 40, 32, 32, 3, 3, 1, 1, 4},     {1, 47, 40, 64, 32, 3, 3, 1, 1, 2},   {3, 9, 11, 16, 16, 1, 1, 0, 0, 8},
+        {2, 32, 32, 3, 32, 5, 5, 2, 2, 8},      {1, 12, 12, 32, 136, 3, 3, 1, 1, 8},  {1, 14, 22, 32, 32, 3, 3, 1, 1, 2},
+        {1, 16, 16, 32, 64, 3, 3, 1, 1, 8},     {2, 20, 36, 32, 64, 3, 3, 1, 1, 8},   {1, 17, 40, 64, 128, 7, 7, 3, 3, 8},
+        {1, 9, 24, 128, 96, 3, 3, 1, 1, 4},     {1, 9, 24, 128, 96, 3, 3, 1, 1, 2},   {2, 3, 3, 32, 32, 3, 3, 1, 1, 8},
+        {1, 16, 16, 64, 64, 3, 3, 1, 1, 8},     {1, 24, 40, 32, 32, 5, 5, 2, 2, 8},   {3, 18, 18, 16, 16, 3, 3, 0, 0, 8},
+    };
+    for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 0);
+    for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 1);
+    std::printf("fails=%d\n", fails);
+    return fails ? 1 : 0;
+}
