@@ -12,7 +12,7 @@ uint32_t round_up(uint32_t v, uint32_t a) { return (v + a - 1) / a * a; }
 size_t round_up_sz(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 // Shared-memory bytes of the barriers and the words after them (see the kernel).
-constexpr uint32_t kBarBytes = (4 * win::kMaxStages + 2 * win::kMaxSlots + 2) * 8 + sizeof(win::Misc);
+constexpr uint32_t kBarBytes = (4 * win::kMaxStages + 2 * win::kMaxSlots + 3) * 8 + sizeof(win::Misc);
 
 // Strips per tile: two unless the image is at most 8 columns wide, or the
 // second strip of a tile would compute more than 15 % extra columns.
@@ -52,7 +52,10 @@ WinPlan plan_conv_win(const ConvShape &s)
     if (p.nch_max > 16) return p;
     const int s_pref = strips_per_tile(s.ow);
     for (int S : {s_pref, 3 - s_pref}) {
-        if (S * p.nch_max * p.nt > 512) continue;  // one slot of accumulators in TMEM
+        // the kernel takes the fewest chunks the filters allow (MMAs that accumulate
+        // into one TMEM buffer issue back to back at the full rate)
+        const int nmin = 1;
+        if (S * std::max(nmin, p.nch_max) * p.nt > 512) continue;  // one slot of accumulators in TMEM
         const int sp = win::kCols * S + s.kw - 1, wh = win::kRows + s.kh - 1;
         if (wh * sp > win::kMaxKP * 128) continue;  // converter positions per thread
         const int tiles_x = (s.ow + win::kCols * S - 1) / (win::kCols * S);
@@ -72,12 +75,19 @@ WinPlan plan_conv_win(const ConvShape &s)
         const uint32_t chunk_stride = p_alloc * 16;
         const uint32_t stage_bytes = chunk_stride * p.groups;
         const uint32_t b_bytes = static_cast<uint32_t>(p.taps * p.groups * p.nt * 16);
-        // rec0, rec1 (16 bytes each), compact direct constants (8), direct flags (1 per 16 channels)
-        const uint32_t rec_bytes = round_up(static_cast<uint32_t>(2 * p.nt * 16 + p.nt * 8 + p.nt / 16), 16);
+        // rec0, rec1 (16 bytes each), direct flags (1 per 16 channels)
+        const uint32_t rec_bytes = round_up(static_cast<uint32_t>(2 * p.nt * 16 + p.nt / 16), 16);
         const uint32_t thr_bytes = s.thr ? static_cast<uint32_t>(p.nt * kThrStride * 4) : 0u;
         const uint32_t tap_bytes = round_up(static_cast<uint32_t>((p.taps + 3) * p.nt * 4), 16);
+        const uint32_t mtab_bytes = round_up(static_cast<uint32_t>(S * p.taps * p.ksteps * 8), 16);
+        const uint32_t pre_bytes = 4096u + static_cast<uint32_t>(p.nt) * 32u;  // pre-load MMA operands
+        // the packed filters are bulk-copied into shared memory when they are whole 16-byte units and fit
+        const long long wraw = static_cast<long long>(s.m) * p.taps * cb;
         bool placed = false;
-        for (int as : {3, 2}) {
+        for (int copy_w : {1, 0}) {
+          if (copy_w && (wraw % 16 != 0 || wraw > 96 * 1024)) continue;
+          const uint32_t wraw_bytes = copy_w ? static_cast<uint32_t>(wraw) : 0u;
+          for (int as : {3, 2}) {
             for (int rs : {3, 2}) {
                 uint32_t off = 0;
                 const uint32_t off_b = off;
@@ -92,10 +102,20 @@ WinPlan plan_conv_win(const ConvShape &s)
                 off += thr_bytes;
                 const uint32_t off_tap = off;
                 off += tap_bytes;
+                const uint32_t off_mtab = round_up(off, 16);
+                off = off_mtab + mtab_bytes;
+                const uint32_t off_pre = round_up(off, 128);
+                off = off_pre + pre_bytes;
+                const uint32_t off_wraw = round_up(off, 128);
+                off = off_wraw + wraw_bytes;
                 const uint32_t off_bar = round_up(off, 16);
                 const uint32_t total = off_bar + kBarBytes;
                 // descriptor start addresses are 14-bit fields of 16-byte units (256 KB)
                 if (total > static_cast<uint32_t>(win::kSmemLimit)) continue;
+                p.off_mtab = off_mtab;
+                p.off_pre = off_pre;
+                p.off_wraw = off_wraw;
+                p.wraw_bytes = wraw_bytes;
                 p.a_stages = as;
                 p.raw_stages = rs;
                 p.off_b = off_b;
@@ -110,9 +130,12 @@ WinPlan plan_conv_win(const ConvShape &s)
                 break;
             }
             if (placed) break;
+          }
+          if (placed) break;
         }
         if (!placed) continue;
         p.s = S;
+        p.nch_min = nmin;
         p.sp = sp;
         p.wh = wh;
         p.p_alloc = static_cast<int>(p_alloc);
@@ -176,6 +199,7 @@ cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvP
     a.raw_stages = plan.raw_stages;
     a.a_stages = plan.a_stages;
     a.nch_max = plan.nch_max;
+    a.nch_min = plan.nch_min;
     a.raw_row_bytes = plan.raw_row_bytes;
     a.raw_bytes = plan.raw_bytes;
     a.chunk_stride = plan.chunk_stride;
@@ -187,11 +211,13 @@ cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvP
     a.off_thr = plan.off_thr;
     a.off_tap = plan.off_tap;
     a.off_bar = plan.off_bar;
+    a.off_mtab = plan.off_mtab;
+    a.off_pre = plan.off_pre;
+    a.off_wraw = plan.off_wraw;
+    a.wraw_bytes = plan.wraw_bytes;
     a.pool = s.pool;
     a.pool_oh = s.oh / 2;
     a.pool_ow = s.ow / 2;
-    for (int i = 0; i < s.kh; ++i)
-        for (int j = 0; j < s.kw; ++j) a.tap_a16[i * s.kw + j] = static_cast<uint32_t>(i * plan.sp + j);
     a.status = device_status_ptr();
     if (!a.status) return cudaErrorInvalidSymbol;
     const long long sms = device_sm_count();

@@ -20,7 +20,9 @@
 // Exactness on fp16 / e4m3 tensor cores (there is no integer tcgen05 MMA on
 // this GPU).  INT-8 activations are staged as x - 128 in fp16, INT-4 / INT-2
 // as themselves in e4m3; weights as themselves; all exact.  Every accumulator
-// is pre-loaded with 1.5 * 2^23, so while the partial sums of a chunk stay
+// starts at 1.5 * 2^23, written by one fp16 MMA that overwrites it with
+// 2048 * 6144 (both exact in fp16, their product exact in fp32) ahead of the
+// layer's MMAs, so no TMEM store is needed; while the partial sums of a chunk stay
 // within 2^22 of it every one is an integer that fp32 holds exactly; the bit
 // pattern minus the pre-load is the chunk's integer sum.  The kernel derives
 // the number of chunks from the filters themselves: the fewest contiguous tap
@@ -28,17 +30,17 @@
 // every output channel (the worst case over all filters is the planner's
 // nch_max, always valid).
 //
-// Filters in the kernel.  The epilogue warps start by reading the packed
-// filters and per-channel constants and writing the B operand (K-major
-// core matrices) and the compression records into shared memory, while the
-// loader and converter warps stage the first windows.  So one qconv_hwc call
-// is one launch and needs no workspace.
+// Filters in the kernel.  The loader first bulk-copies the packed filters and
+// the first windows' input rows; meanwhile the whole block turns the filters
+// into the B operand (K-major core matrices), derives the per-channel
+// compression records, the chunk count and the MMA issue order, all in shared
+// memory.  So one qconv_hwc call is one launch and needs no workspace.
 //
-// Warp roles (one persistent CTA per SM, 14 warps):
+// Warp roles after that (one persistent CTA per SM, 14 warps):
 //   warps 0-3   converters: raw window -> staged operand, every position
-//   warps 4-11  filter preparation, then epilogue: warp w reads TMEM lane
-//               quarter w % 4 and one half of the output channels; sums the
-//               chunks, compresses, packs at Q bits and stores
+//   warps 4-11  epilogue: warp w reads TMEM lane quarter w % 4 and one half
+//               of the output channels; sums the chunks, compresses, packs at
+//               Q bits and stores
 //   warp 12     MMA issue (converged warp, elected lane)
 //   warp 13     bulk copies of the input rows of each window
 // Every wait is bounded; on a timeout the kernel records QNN_ETIMEOUT in the
@@ -64,14 +66,16 @@ constexpr int kMaxKP = 5;             // window positions per converter thread a
 constexpr int kSmemLimit = 232448;    // 227 KB opt-in dynamic shared memory per block
 
 // Shared-memory words after the barriers: the TMEM base, the chunk count the
-// filters allow, the accumulator slot count and width, the chunk-mask vote.
+// filters allow, the accumulator slot count and width, the chunk-mask vote,
+// the MMAs per tile.
 struct Misc {
     uint32_t tmem;
     uint32_t nch;
     uint32_t nslots;
     uint32_t slot_cols;
     uint32_t mask;
-    uint32_t pad[3];
+    uint32_t nmma;  // MMAs per tile (entries of the issue table)
+    uint32_t pad[2];
 };
 
 struct WinArgs {
@@ -90,12 +94,14 @@ struct WinArgs {
     int full_rows;
     int tiles_x, tiles_per_img, total_tiles;
     FastDiv fd_tpi, fd_tx, fd_sp;
-    int raw_stages, a_stages, nch_max;
+    int raw_stages, a_stages, nch_max, nch_min;
     uint32_t raw_row_bytes, raw_bytes, chunk_stride, stage_bytes;
     uint32_t off_b, off_a, off_raw, off_rec, off_thr, off_tap, off_bar;
+    uint32_t off_wraw, wraw_bytes;  // packed filters copied into shared memory (0 bytes: read from global)
+    uint32_t off_mtab;              // the MMA issue table (S * taps * ksteps entries of 8 bytes)
+    uint32_t off_pre;               // operands of the pre-load MMA (A 4 KB, then B 2 * NT * 16 bytes)
     int pool, pool_oh, pool_ow;
     int *status;
-    uint32_t tap_a16[kMaxTaps];  // per tap (i, j): window position i * sp + j
 };
 
 // Tile t: image, first output row and column, window origin in the input.
@@ -130,71 +136,101 @@ __device__ __forceinline__ int col_hi(const WinArgs &a, const Geo &g)
 
 // ---------------------------------------------------------------- loader (warp 13)
 
-// The input rows of each tile's window: one bulk copy when windows span whole
-// image rows, else one per row (lanes issue them in parallel).
-__device__ __forceinline__ void loader_role(const WinArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty)
+// The loader's position in its ring of raw windows.
+struct LoadState {
+    int rs, issued, t;
+    uint32_t ph;
+};
+
+// The packed filters, copied into shared memory for the filter preparation.
+__device__ __forceinline__ void load_filters(const WinArgs &a, uint8_t *smem, uint64_t *w_full)
+{
+    if (a.wraw_bytes && (threadIdx.x & 31) == 0) {
+        mbar_arrive_expect_tx(w_full, a.wraw_bytes);
+        for (uint32_t off = 0; off < a.wraw_bytes; off += 32768u)
+            bulk_g2s(smem + a.off_wraw + off, a.w + off, min(32768u, a.wraw_bytes - off), w_full);
+    }
+    __syncwarp();
+}
+
+// The input rows of up to `count` more tiles' windows: one bulk copy when
+// windows span whole image rows, else one per row (lanes issue them in
+// parallel).
+__device__ __forceinline__ void load_windows(const WinArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
+                                             LoadState &st, int count)
 {
     const int lane = threadIdx.x & 31;
-    int rs = 0, issued = 0;
-    uint32_t ph = 0;
-    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
-        const Geo g = geo_of(a, t);
+    for (; st.t < a.total_tiles && count > 0; st.t += gridDim.x, --count) {
+        const Geo g = geo_of(a, st.t);
         const int r0 = row_lo(a, g), r1 = row_hi(a, g);
         const int c0 = col_lo(a, g), c1 = col_hi(a, g);
-        if (!mbar_wait_warp(&raw_empty[rs], ph ^ 1u, a.status)) break;
-        uint8_t *dst = smem + a.off_raw + rs * a.raw_bytes;
+        if (!mbar_wait_warp(&raw_empty[st.rs], st.ph ^ 1u, a.status)) {
+            st.t = a.total_tiles;  // give up: the other roles time out as well
+            break;
+        }
+        uint8_t *dst = smem + a.off_raw + st.rs * a.raw_bytes;
         const int rows = r1 - r0;
         if (a.full_rows) {
             const uint32_t bytes = static_cast<uint32_t>(rows) * a.raw_row_bytes;
             if (lane == 0) {
-                mbar_arrive_expect_tx(&raw_full[rs], bytes);
+                mbar_arrive_expect_tx(&raw_full[st.rs], bytes);
                 const uint8_t *src = a.x + (static_cast<long long>(g.img) * a.h + (g.iy0 + r0)) * a.raw_row_bytes;
                 for (uint32_t off = 0; off < bytes; off += 32768u)
-                    bulk_g2s(dst + off, src + off, min(32768u, bytes - off), &raw_full[rs]);
+                    bulk_g2s(dst + off, src + off, min(32768u, bytes - off), &raw_full[st.rs]);
             }
         } else {
             const uint32_t seg = static_cast<uint32_t>(c1 - c0) * a.cb;  // cb is a multiple of 16 here
-            if (lane == 0) mbar_arrive_expect_tx(&raw_full[rs], seg * static_cast<uint32_t>(rows));
+            if (lane == 0) mbar_arrive_expect_tx(&raw_full[st.rs], seg * static_cast<uint32_t>(rows));
             __syncwarp();
             if (seg)
                 for (int r = r0 + lane; r < r1; r += 32) {
                     const uint8_t *src =
                         a.x + ((static_cast<long long>(g.img) * a.h + (g.iy0 + r)) * a.w_ + (g.ix0 + c0)) * a.cb;
-                    bulk_g2s(dst + (r - r0) * a.raw_row_bytes, src, seg, &raw_full[rs]);
+                    bulk_g2s(dst + (r - r0) * a.raw_row_bytes, src, seg, &raw_full[st.rs]);
                 }
         }
         __syncwarp();
-        ++issued;
-        if (++rs == a.raw_stages) {
-            rs = 0;
-            ph ^= 1u;
+        ++st.issued;
+        if (++st.rs == a.raw_stages) {
+            st.rs = 0;
+            st.ph ^= 1u;
         }
     }
-    // every copy lands before the block exits
-    for (int k = 0; k < a.raw_stages && k < issued; ++k) {
-        if (--rs < 0) {
-            rs = a.raw_stages - 1;
-            ph ^= 1u;
+}
+
+// Every copy lands before the block exits.
+__device__ __forceinline__ void load_drain(const WinArgs &a, uint64_t *raw_full, uint64_t *w_full, LoadState st)
+{
+    for (int k = 0; k < a.raw_stages && k < st.issued; ++k) {
+        if (--st.rs < 0) {
+            st.rs = a.raw_stages - 1;
+            st.ph ^= 1u;
         }
-        mbar_wait_warp(&raw_full[rs], ph, a.status);
+        mbar_wait_warp(&raw_full[st.rs], st.ph, a.status);
     }
+    if (a.wraw_bytes) mbar_wait_warp(w_full, 0, a.status);
 }
 
 // ---------------------------------------------------------------- converters (warps 0-3)
 
-// Staged encoding of 8 (fp16) or 16 (e4m3) channels of one pixel.
+// Staged encoding of one K-chunk of a pixel from its packed bytes: 8 unsigned
+// bytes -> 8 fp16 (x - 128), or 16 nibbles / crumbs -> 16 e4m3 (the channel
+// orders of cvt_raw_f8, which the filter layout follows).
 template <int BITS>
-__device__ __forceinline__ uint4 stage_cvt(const uint8_t *p)
+__device__ __forceinline__ uint4 stage_chunk(uint2 v)
 {
-    if (BITS == 8) return cvt_u8x8(*reinterpret_cast<const uint2 *>(p));
-    return cvt_raw_f8<BITS>(p);
+    if (BITS == 8) return cvt_u8x8(v);
+    if (BITS == 4) return make_uint4(e4m3x4(v.x), e4m3x4(v.x >> 16), e4m3x4(v.y), e4m3x4(v.y >> 16));
+    const uint32_t ev = v.x & 0x33333333u, od = (v.x >> 2) & 0x33333333u;  // crumbs 2k and 2k+1 as nibbles
+    return make_uint4(e4m3x4(ev), e4m3x4(od), e4m3x4(ev >> 16), e4m3x4(od >> 16));
 }
 
-// Every position of the tile's window, K-chunk plane by plane: the staged
-// value of the input pixel there, or the encoded zero outside the image and
-// past the channel count.  Thread t owns positions t, t + 128, ... of every
-// plane (their window row and column are decoded once per kernel), so a
-// warp's stores are consecutive 16-byte positions.
+// Every position of the tile's window: the staged value of the input pixel
+// there, or the encoded zero outside the image and past the channel count.
+// Thread t owns positions t, t + 128, ...; per position it loads the pixel's
+// packed channels (16-byte loads when a pixel is a whole number of 16-byte
+// units, else 8-byte ones) and stores one 16-byte chunk per K-chunk plane, so
+// a warp's stores are consecutive positions of a plane.
 template <int BITS>
 __device__ __forceinline__ void converter_role(const WinArgs &a, uint8_t *smem, uint64_t *raw_full, uint64_t *raw_empty,
                                                uint64_t *a_full, uint64_t *a_empty)
@@ -202,15 +238,10 @@ __device__ __forceinline__ void converter_role(const WinArgs &a, uint8_t *smem, 
     constexpr uint32_t kPad = BITS == 8 ? 0xD800D800u : 0u;  // fp16 -128.0 (x = 0), e4m3 0
     constexpr int kGroupBytes = BITS == 8 ? 8 : 16 * BITS / 8;  // packed bytes of one K-chunk
     const int tid = threadIdx.x;
-    int pr[kMaxKP], pc[kMaxKP];
-#pragma unroll
-    for (int k = 0; k < kMaxKP; ++k) {
-        const int pos = tid + 128 * k;
-        pr[k] = fdiv(pos, a.fd_sp);
-        pc[k] = pos - pr[k] * a.sp;
-        if (pos >= a.npos) pr[k] = -1;  // no position
-    }
     const int cgroups = a.c * BITS / 8 / kGroupBytes;  // K-chunks that hold input channels (c is a multiple of kch)
+    const int groups = a.groups;
+    const int words = a.cb / 8;             // 8-byte words of one pixel (at most 8)
+    const bool wide = (a.cb & 15) == 0;     // 16-byte aligned pixels
     int rs = 0, as = 0;
     uint32_t r_ph = 0, a_ph = 0;
     for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
@@ -220,33 +251,56 @@ __device__ __forceinline__ void converter_role(const WinArgs &a, uint8_t *smem, 
         // raw column of window column px: the copied span starts at window column c0
         // (whole rows start at image column 0, i.e. window column -ix0)
         const int base_col = a.full_rows ? g.ix0 : -c0;
-        uint32_t src[kMaxKP];
-        bool ok[kMaxKP];
-#pragma unroll
-        for (int k = 0; k < kMaxKP; ++k) {
-            ok[k] = pr[k] >= r0 && pr[k] < r1 && pc[k] >= c0 && pc[k] < c1;
-            src[k] = ok[k] ? static_cast<uint32_t>(pr[k] - r0) * a.raw_row_bytes +
-                                 static_cast<uint32_t>((pc[k] + base_col) * a.cb)
-                           : 0u;
-        }
         if (!mbar_wait_warp(&raw_full[rs], r_ph, a.status)) return;
         if (!mbar_wait_warp(&a_empty[as], a_ph ^ 1u, a.status)) return;
         const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
         const uint32_t stage = smem_addr(smem + a.off_a + as * a.stage_bytes);
-        for (int gq = 0; gq < a.groups; ++gq) {
-            const bool has = gq < cgroups;
-            uint4 v[kMaxKP];
+        // Three positions per iteration, every load of the three issued before any
+        // conversion (shared memory is busy with the tensor cores' operand reads,
+        // so each round trip is long); one loop body keeps the code of the four
+        // roles running side by side on each SM sub-partition small.
+#pragma unroll 1
+        for (int pos0 = tid; pos0 < a.npos; pos0 += 3 * 128) {
+            uint2 pv[3][8];
+            bool ok[3];
 #pragma unroll
-            for (int k = 0; k < kMaxKP; ++k) {
-                // every load is issued (a safe address where the value is padding)
-                const uint8_t *q = raw + ((ok[k] && has) ? src[k] + gq * kGroupBytes : 0u);
-                const uint4 x = stage_cvt<BITS>(q);
-                v[k] = (ok[k] && has) ? x : make_uint4(kPad, kPad, kPad, kPad);
+            for (int u = 0; u < 3; ++u) {
+                const int pos = pos0 + u * 128;
+                const int pr = fdiv(pos, a.fd_sp), pc = pos - pr * a.sp;
+                ok[u] = pos < a.npos && pr >= r0 && pr < r1 && pc >= c0 && pc < c1;
+                // the pixel's packed channels (a safe address where the value is padding)
+                const uint8_t *q = raw + (ok[u] ? static_cast<uint32_t>(pr - r0) * a.raw_row_bytes +
+                                                      static_cast<uint32_t>((pc + base_col) * a.cb)
+                                                : 0u);
+                if (wide) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const uint4 v = 2 * j < words ? *reinterpret_cast<const uint4 *>(q + 16 * j) : make_uint4(0, 0, 0, 0);
+                        pv[u][2 * j] = make_uint2(v.x, v.y);
+                        pv[u][2 * j + 1] = make_uint2(v.z, v.w);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        pv[u][j] = j < words ? *reinterpret_cast<const uint2 *>(q + 8 * j) : make_uint2(0, 0);
+                }
             }
-            const uint32_t plane = stage + gq * a.chunk_stride;
 #pragma unroll
-            for (int k = 0; k < kMaxKP; ++k)
-                if (pr[k] >= 0) sts128(plane + static_cast<uint32_t>(tid + 128 * k) * 16u, v[k]);
+            for (int u = 0; u < 3; ++u) {
+                const int pos = pos0 + u * 128;
+                if (pos >= a.npos) break;
+                const uint32_t pos16 = static_cast<uint32_t>(pos) * 16u;
+#pragma unroll
+                for (int gq = 0; gq < 8; ++gq) {
+                    if (gq >= groups) break;
+                    uint2 v;
+                    if (kGroupBytes == 8) v = pv[u][gq];
+                    else v = make_uint2((gq & 1) ? pv[u][gq >> 1].y : pv[u][gq >> 1].x, 0u);
+                    const uint4 x = stage_chunk<BITS>(v);
+                    const bool real = ok[u] && gq < cgroups;
+                    sts128(stage + gq * a.chunk_stride + pos16, real ? x : make_uint4(kPad, kPad, kPad, kPad));
+                }
+            }
         }
         fence_proxy_async_smem();
         mbar_arrive(&a_full[as]);
@@ -264,14 +318,47 @@ __device__ __forceinline__ void converter_role(const WinArgs &a, uint8_t *smem, 
 
 // ---------------------------------------------------------------- MMA issue (warp 12)
 
+__device__ __forceinline__ uint64_t desc_of(uint32_t lo, uint32_t hi)
+{
+    return (static_cast<uint64_t>(hi) << 32) | lo;
+}
+
+template <bool F8>
+__device__ __forceinline__ void mma_nc(uint32_t d, uint64_t ad, uint64_t bd, uint32_t idesc)
+{
+    if (F8) mma_f8_ss_warp_nc(d, ad, bd, idesc, 1u);
+    else mma_f16_ss_warp_nc(d, ad, bd, idesc, 1u);
+}
+
+// One tile's MMAs with every offset known at compile time (one exact chunk,
+// KH x KW taps, KS k-steps per tap, S strips): a descriptor is its template's
+// low word plus an offset (a start address field that cannot carry out of its
+// 14 bits), so each MMA costs an addition or two and the issue.
+template <int KH, int KW, int KS, int S, int NT, bool F8>
+__device__ __forceinline__ void issue_fixed(uint32_t d0, uint32_t alo, uint32_t ahi, uint32_t blo, uint32_t bhi,
+                                            uint32_t idesc, int sp, uint32_t kstep_a)
+{
+    // one kernel row per iteration: its KW * KS * S MMAs unrolled
+#pragma unroll 1
+    for (int i = 0; i < KH; ++i) {
+        const uint32_t arow = alo + static_cast<uint32_t>(i * sp);
+#pragma unroll
+        for (int j = 0; j < KW; ++j)
+#pragma unroll
+            for (int kk = 0; kk < KS; ++kk) {
+                const uint64_t bd = desc_of(blo + static_cast<uint32_t>(((i * KW + j) * 2 * KS + 2 * kk) * NT), bhi);
+#pragma unroll
+                for (int s = 0; s < S; ++s)
+                    mma_nc<F8>(d0 + s * NT, desc_of(arow + j + kk * kstep_a + s * kCols, ahi), bd, idesc);
+            }
+    }
+}
+
 template <int NT, bool F8>
 __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64_t *a_full, uint64_t *a_empty,
-                                         uint64_t *acc_full, uint64_t *acc_empty, uint64_t *b_ready, uint64_t *done,
-                                         const volatile Misc *misc)
+                                         uint64_t *acc_full, uint64_t *acc_empty, uint64_t *done, const Misc *misc)
 {
     int *const status = a.status;
-    bool ok = mbar_wait_warp(b_ready, 0, status);
-    tc_fence_after();
     const uint32_t tmem = misc->tmem;
     const int nch = static_cast<int>(misc->nch), nslots = static_cast<int>(misc->nslots);
     const uint32_t slot_cols = misc->slot_cols;
@@ -280,30 +367,48 @@ __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64
     const uint64_t b_tmpl = smem_desc(0, NT * 16, 128);
     const uint32_t b16 = smem_addr(smem + a.off_b) >> 4;
     const uint32_t stages16 = smem_addr(smem + a.off_a) >> 4;
-    const uint32_t kstep_a = 2u * (a.chunk_stride >> 4), kstep_b = 2u * NT;
-    const uint32_t tap_b = static_cast<uint32_t>(a.groups) * NT;
-    const int ct = (a.taps + nch - 1) / nch;  // taps per chunk
-    const int ksteps = a.ksteps, S = a.s;
-    for (int i = 0, t = blockIdx.x; ok && t < a.total_tiles; ++i, t += gridDim.x) {
+    const uint32_t kstep_a = 2u * (a.chunk_stride >> 4);
+    // the pre-load MMA: fp16 operands in shared memory, accumulate = 0
+    const uint32_t pre16 = smem_addr(smem + a.off_pre) >> 4;
+    const uint64_t pre_a = smem_desc(0, 2048, 128) + pre16;
+    const uint64_t pre_b = smem_desc(0, NT * 16, 128) + pre16 + 256;
+    const int nacc = a.s * nch;
+    // the issue order (built by the filter preparation): one 8-byte entry per MMA,
+    // {A offset in 16-byte units | accumulator column << 16, B offset}
+    const uint2 *tab = reinterpret_cast<const uint2 *>(smem + a.off_mtab);
+    const int nu = static_cast<int>(misc->nmma);
+    // the common shapes with one exact chunk issue from unrolled code
+    const int fixed = nch != 1 ? 0
+                      : (a.kh == 3 && a.kw == 3 && a.ksteps == 2 && a.s == 2) ? 1
+                      : (a.kh == 3 && a.kw == 3 && a.ksteps == 1 && a.s == 2) ? 2
+                      : (a.kh == 5 && a.kw == 5 && a.ksteps == 2 && a.s == 2) ? 3
+                      : (a.kh == 5 && a.kw == 5 && a.ksteps == 2 && a.s == 1) ? 4
+                      : (a.kh == 3 && a.kw == 3 && a.ksteps == 4 && a.s == 2) ? 5
+                                                                                : 0;
+    for (int i = 0, t = blockIdx.x; t < a.total_tiles; ++i, t += gridDim.x) {
         const int as = i % a.a_stages, slot = i % nslots;
         if (!mbar_wait_warp(&a_full[as], (i / a.a_stages) & 1, status)) break;
         if (!mbar_wait_warp(&acc_empty[slot], (i / nslots) & 1, status)) break;
         tc_fence_after();
-        const uint32_t abase = stages16 + as * (a.stage_bytes >> 4);
-        for (int s = 0; s < S; ++s) {
-            for (int c = 0; c < nch; ++c) {
-                const uint32_t d = tmem + slot * slot_cols + static_cast<uint32_t>(s * nch + c) * NT;
-                const int t1 = min(a.taps, (c + 1) * ct);
-#pragma unroll 2
-                for (int tap = c * ct; tap < t1; ++tap) {
-                    const uint64_t ad = a_tmpl + (abase + a.tap_a16[tap] + s * kCols);
-                    const uint64_t bd = b_tmpl + (b16 + tap * tap_b);
-                    for (int kk = 0; kk < ksteps; ++kk) {
-                        if (F8) mma_f8_ss_warp(d, ad + kk * kstep_a, bd + kk * kstep_b, idesc, 1u);
-                        else mma_f16_ss_warp(d, ad + kk * kstep_a, bd + kk * kstep_b, idesc, 1u);
-                    }
+        const uint64_t abase = a_tmpl + (stages16 + as * (a.stage_bytes >> 4));
+        const uint64_t bbase = b_tmpl + b16;
+        const uint32_t d0 = tmem + slot * slot_cols;
+        // every accumulator of the slot starts at the pre-load (accumulate = 0)
+        for (int b = 0; b < nacc; ++b) mma_f16_ss_warp_nc(d0 + b * NT, pre_a, pre_b, idesc, 0u);
+        const uint32_t alo = static_cast<uint32_t>(abase), ahi = static_cast<uint32_t>(abase >> 32);
+        const uint32_t blo = static_cast<uint32_t>(bbase), bhi = static_cast<uint32_t>(bbase >> 32);
+        switch (fixed) {
+            case 1: issue_fixed<3, 3, 2, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 2: issue_fixed<3, 3, 1, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 3: issue_fixed<5, 5, 2, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 4: issue_fixed<5, 5, 2, 1, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 5: issue_fixed<3, 3, 4, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            default:
+#pragma unroll 4
+                for (int u = 0; u < nu; ++u) {
+                    const uint2 e = tab[u];
+                    mma_nc<F8>(d0 + (e.x >> 16), abase + (e.x & 0xFFFFu), bbase + e.y, idesc);
                 }
-            }
         }
         mma_commit_warp(&acc_full[slot]);
         mma_commit_warp(&a_empty[as]);
@@ -313,36 +418,33 @@ __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64
     mbar_wait_warp(done, 0, status);
 }
 
-// ---------------------------------------------------------------- filter preparation (warps 4-11)
+// ---------------------------------------------------------------- filter preparation (the whole block)
 
-// Epilogue barrier (named barrier 1, the eight epilogue warps).
-__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory"); }
-
-// One K-chunk of one output channel's filter at one tap: the staged B row
-// (8 fp16 or 16 e4m3 values in the converter's channel order) and the sums
-// the compression constants and the chunk count need.
+// One K-chunk of one output channel's filter at one tap, from its packed
+// bytes (8, or 4 at INT-2, in v): the staged B row (8 fp16 or 16 e4m3 values
+// in the converter's channel order) and the sums the compression constants and
+// the chunk count need.
 template <int BITS>
-__device__ __forceinline__ uint4 filter_chunk(const uint8_t *p, bool has, int &sum, int &pos, int &neg, int &abs)
+__device__ __forceinline__ uint4 filter_chunk(uint2 v, int &sum, int &pos, int &neg, int &abs)
 {
-    if (!has) return make_uint4(0u, 0u, 0u, 0u);  // +0 in fp16 and e4m3
     if (BITS == 8) {
-        const uint2 v = *reinterpret_cast<const uint2 *>(p);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int wv = static_cast<int8_t>(((k < 4 ? v.x : v.y) >> (8 * (k & 3))) & 0xFFu);
-            sum += wv;
-            pos += max(wv, 0);
-            neg += min(wv, 0);
-            abs += wv < 0 ? -wv : wv;
-        }
+        // byte sums by 4-way signed dot products with ones: the weights, and their negative parts
+        const int all = __dp4a(static_cast<int>(v.x), 0x01010101, __dp4a(static_cast<int>(v.y), 0x01010101, 0));
+        const int ng = __dp4a(static_cast<int>(__vmins4(v.x, 0u)), 0x01010101,
+                              __dp4a(static_cast<int>(__vmins4(v.y, 0u)), 0x01010101, 0));
+        sum += all;
+        neg += ng;
+        pos += all - ng;
+        abs += all - 2 * ng;
         // byte b ^ 0x80 is the weight plus 128 as an unsigned byte: the activation encoding gives the weight
         return cvt_u8x8(make_uint2(v.x ^ 0x80808080u, v.y ^ 0x80808080u));
     }
     uint8_t e[16];
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
-        constexpr int per = 8 / BITS;
-        const int f = (p[k / per] >> ((k % per) * BITS)) & ((1 << BITS) - 1);
+        constexpr int per = 32 / BITS;  // values per 32-bit word
+        const uint32_t word = k / per == 0 ? v.x : v.y;
+        const int f = (word >> ((k % per) * BITS)) & ((1 << BITS) - 1);
         const int wv = f >= (1 << (BITS - 1)) ? f - (1 << BITS) : f;
         sum += wv;
         pos += max(wv, 0);
@@ -365,40 +467,76 @@ __device__ __forceinline__ uint4 filter_chunk(const uint8_t *p, bool has, int &s
 // rec1 = {beta, ulo, uhi, lambda}, as in the tensor-core prep kernel, with
 // acc + bias = s + beta for the raw chunk sum s) and the accumulator slots.
 template <int BITS, int NT>
-__device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem, Misc *misc, uint64_t *b_ready)
+__device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem, Misc *misc, uint64_t *w_full)
 {
     constexpr int kGroupBytes = BITS == 8 ? 8 : 16 * BITS / 8;
     constexpr int kMaxX = BITS == 8 ? 128 : (1 << BITS) - 1;  // largest |staged activation|
-    const int et = threadIdx.x - kEpiWarp0 * 32;                // 0..255
+    constexpr int kItemThreads = kThreads / NT * NT;            // threads with a filter item: a multiple of NT
+    const int et = threadIdx.x;
     int *tapabs = reinterpret_cast<int *>(smem + a.off_tap);    // [taps][NT]
     int *sums = tapabs + a.taps * NT;                           // [3][NT]: sum, positive part, negative part
-    for (int i = et; i < 3 * NT; i += kEpiWarps * 32) sums[i] = 0;
+    for (int i = et; i < 3 * NT; i += kThreads) sums[i] = 0;
     if (et == 0) misc->mask = ~0u;
-    epi_sync();
-    // item i: channel n = i % NT (fixed per thread: 256 is a multiple of NT), tap i / NT
+    __syncthreads();
+    // item i: channel n = i % NT (fixed per thread: kItemThreads is a multiple of NT), tap i / NT.
+    // Every load of a batch of two items goes out before any of them is used.
     const int cgroups = a.c * BITS / 8 / kGroupBytes;
     int sum = 0, pos = 0, neg = 0;
     const int n = et % NT;
-    for (int i = et; i < a.taps * NT; i += kEpiWarps * 32) {
-        const int tap = i / NT;
-        int abs = 0;
-        const uint8_t *src = a.w + (static_cast<long long>(n) * a.taps + tap) * (a.c * BITS / 8);
-        for (int gq = 0; gq < a.groups; ++gq) {
-            const uint4 v = filter_chunk<BITS>(src + gq * kGroupBytes, n < a.m && gq < cgroups, sum, pos, neg, abs);
-            *reinterpret_cast<uint4 *>(smem + a.off_b + ((tap * a.groups + gq) * NT + n) * 16) = v;
+    const int items = a.taps * NT;
+    const long long wrow = static_cast<long long>(a.c) * BITS / 8;  // packed bytes of one tap of one filter
+    // the packed filters: the loader's shared-memory copy, or global memory
+    const bool copied = a.wraw_bytes != 0;
+    if (copied) mbar_wait_warp(w_full, 0, a.status);
+    const uint8_t *wsrc = copied ? smem + a.off_wraw : a.w;
+    for (int i0 = et; et < kItemThreads && i0 < items; i0 += 2 * kItemThreads) {
+        uint2 raw[2][8];
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+            const int i = i0 + b * kItemThreads;
+            const uint8_t *src = wsrc + (static_cast<long long>(n) * a.taps + i / NT) * wrow;
+#pragma unroll
+            for (int gq = 0; gq < 8; ++gq) {
+                const bool has = i < items && n < a.m && gq < cgroups;
+                if (kGroupBytes == 8) {
+                    const uint2 *q = reinterpret_cast<const uint2 *>(src + gq * 8);
+                    raw[b][gq] = !has ? make_uint2(0u, 0u) : copied ? *q : __ldg(q);
+                } else {
+                    const uint32_t *q = reinterpret_cast<const uint32_t *>(src + gq * 4);
+                    raw[b][gq] = make_uint2(!has ? 0u : copied ? *q : __ldg(q), 0u);
+                }
+            }
         }
-        tapabs[tap * NT + n] = abs;
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+            const int i = i0 + b * kItemThreads;
+            if (i >= items) break;
+            const int tap = i / NT;
+            int abs = 0;
+#pragma unroll
+            for (int gq = 0; gq < 8; ++gq) {
+                if (gq >= a.groups) break;
+                // K-chunks past the channel count (and filters past m) stage +0
+                const uint4 v = (n < a.m && gq < cgroups) ? filter_chunk<BITS>(raw[b][gq], sum, pos, neg, abs)
+                                                         : make_uint4(0u, 0u, 0u, 0u);
+                *reinterpret_cast<uint4 *>(smem + a.off_b + ((tap * a.groups + gq) * NT + n) * 16) = v;
+            }
+            tapabs[tap * NT + n] = abs;
+        }
     }
-    if (a.taps * NT > et) {  // this thread saw channel n
+    if (et < kItemThreads && items > et) {  // this thread saw channel n
         atomicAdd(&sums[n], sum);
         atomicAdd(&sums[NT + n], pos);
         atomicAdd(&sums[2 * NT + n], neg);
     }
-    epi_sync();
-    // chunk counts c = 1 .. nch_max whose even tap split keeps every chunk exact
+    __syncthreads();
+    // Chunk counts c in [nch_min, c_force] whose even tap split has no empty
+    // chunk and keeps every chunk of every channel exact; c_force = max(nch_min,
+    // nch_max) holds by the planner's worst-case bound whatever the filters.
+    const int c_force = max(a.nch_min, a.nch_max);
     if (et < NT) {
         uint32_t okmask = 0;
-        for (int c = 1; c <= a.nch_max; ++c) {
+        for (int c = a.nch_min; c <= c_force; ++c) {
             const int ct = (a.taps + c - 1) / c;
             if ((c - 1) * ct >= a.taps) continue;  // an empty chunk: not a c-chunk split
             bool good = true;
@@ -409,10 +547,10 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
             }
             if (good) okmask |= 1u << c;
         }
-        okmask |= 1u << a.nch_max;  // valid for any filters by the planner's bound
+        okmask |= 1u << c_force;
         atomicAnd(&misc->mask, okmask);
     }
-    epi_sync();
+    __syncthreads();
     const int nch = __ffs(static_cast<int>(misc->mask)) - 1;
     // per-channel records
     int4 *rec0 = reinterpret_cast<int4 *>(smem + a.off_rec);
@@ -450,90 +588,137 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
         rec0[o] = r0;
         rec1[o] = r1;
     }
-    epi_sync();
-    // compact direct-mode constants, and one "all direct" flag per 16-channel group
-    uint2 *dcon = reinterpret_cast<uint2 *>(rec1 + NT);
-    uint8_t *gd = reinterpret_cast<uint8_t *>(dcon + NT);
-    if (et < NT) {
-        const int4 r0 = rec0[et];
-        dcon[et] = make_uint2(static_cast<uint32_t>(r0.x),
-                              (static_cast<uint32_t>(r0.y) & 0xFFFFu) | (static_cast<uint32_t>(r0.z) << 16));
-    }
+    __syncthreads();
+    // one "all direct" flag per 16-channel group
+    uint8_t *gd = reinterpret_cast<uint8_t *>(rec1 + NT);
     if (et < NT / 16) {
         int all = 1;
         for (int k = 0; k < 16; ++k) all &= rec0[et * 16 + k].w == kModeDirect;
         gd[et] = static_cast<uint8_t>(all);
     }
-    // B was written through the generic proxy; the tensor cores read it through the async proxy
+    // The MMA issue order, one 8-byte entry per MMA: {A offset (16-byte units
+    // within a stage) | accumulator column << 16, B offset}.  The accumulators
+    // (chunk c, strip s) are independent and consecutive MMAs go to different
+    // ones, so the tensor pipe does not wait on the previous MMA's accumulator:
+    // the k-th step of every chunk and strip goes out together.  Thread et
+    // writes the entries of step pair (jt, kk) = (et / ksteps, et % ksteps);
+    // only the last chunk is shorter (last_len taps).
+    const int ct = (a.taps + nch - 1) / nch, last_len = a.taps - (nch - 1) * ct;
+    if (et < ct * a.ksteps) {
+        const int jt = et / a.ksteps, kk = et - jt * a.ksteps;
+        const int nj = jt < last_len ? nch : nch - 1;  // chunks with a tap at step jt
+        const int before = jt * nch - max(0, jt - last_len);
+        int u = a.s * (a.ksteps * before + kk * nj);
+        uint2 *tab = reinterpret_cast<uint2 *>(smem + a.off_mtab);
+        const uint32_t kstep_a = 2u * (a.chunk_stride >> 4), kstep_b = 2u * NT;
+        for (int c = 0; c < nj; ++c) {
+            const int tap = c * ct + jt, ti = tap / a.kw, tj = tap - ti * a.kw;
+            for (int s = 0; s < a.s; ++s, ++u)
+                tab[u] = make_uint2((static_cast<uint32_t>(ti * a.sp + tj) + kk * kstep_a + s * kCols) |
+                                        (static_cast<uint32_t>(s * nch + c) * NT << 16),
+                                    static_cast<uint32_t>(tap * a.groups) * NT + kk * kstep_b);
+        }
+    }
+    // Operands of the pre-load MMA (K-major, 8-row core matrices 128 bytes apart,
+    // the second K-chunk 16 rows further): A rows {2048, 0, ...}, B rows {6144, 0, ...},
+    // so every accumulator element becomes 2048 * 6144 = 1.5 * 2^23.
+    {
+        uint32_t *pre = reinterpret_cast<uint32_t *>(smem + a.off_pre);
+        const int aw = 128 * 2 * 4, bw = NT * 2 * 4;  // 32-bit words: A (128 rows, 2 chunks), B (NT rows, 2 chunks)
+        for (int i = et; i < aw + bw; i += kThreads) {
+            const bool is_a = i < aw;
+            const int j = is_a ? i : i - aw;       // word within the operand
+            const int rows = is_a ? 128 : NT;
+            const bool first = j < rows * 4 && (j & 3) == 0;  // chunk 0, element 0 of a row
+            pre[i] = first ? (is_a ? 0x6800u : 0x6E00u) : 0u;  // fp16 2048, 6144
+        }
+    }
+    // B and the pre-load operands were written through the generic proxy; the
+    // tensor cores read them through the async proxy
     fence_proxy_async_smem();
-    epi_sync();
+    __syncthreads();
     if (et == 0) {
         const uint32_t cols = static_cast<uint32_t>(a.s * nch * NT);
         misc->nch = static_cast<uint32_t>(nch);
         misc->slot_cols = cols;
         misc->nslots = min(static_cast<uint32_t>(kMaxSlots), 512u / cols);
-        mbar_arrive(b_ready);
+        misc->nmma = static_cast<uint32_t>(a.s * a.taps * a.ksteps);
     }
-    epi_sync();
+    // the roles start after this barrier: B, the records, the table and the
+    // slot layout are complete
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
 }
 
 // ---------------------------------------------------------------- epilogue (warps 4-11)
 
-template <int CW>
-__device__ __forceinline__ void tmem_fill(uint32_t taddr)
+// The integer sums of the chunks' bit patterns of EB consecutive columns of
+// the tile's strips (chunk buffers `stride` columns apart, strip 1's buffers at
+// a1).  With at most two chunks every load of the block is in flight before one
+// wait.
+template <int EB>
+__device__ __forceinline__ void tmem_load(uint32_t addr, uint32_t (&v)[EB])
 {
-    if (CW == 8) {
-        tmem_st8_fill(taddr, kMagic);
-    } else {
+    if constexpr (EB >= 16) {
 #pragma unroll
-        for (int c = 0; c < CW; c += 16) tmem_st16_fill(taddr + c, kMagic);
+        for (int b0 = 0; b0 < EB; b0 += 16) tmem_ld16(addr + b0, *reinterpret_cast<uint32_t(*)[16]>(v + b0));
+    } else {
+        tmem_ld8(addr, *reinterpret_cast<uint32_t(*)[8]>(v));
     }
 }
 
-// The integer sum of the chunks' bit patterns of EB consecutive columns of one
-// strip (chunk buffers `stride` columns apart), each buffer's columns refilled
-// with the pre-load once read.  NCH > 0: that many chunks, each chunk's loads
-// in flight before one wait; NCH = 0: any count.
-template <int EB, int NCH>
-__device__ __forceinline__ void drain(uint32_t addr, uint32_t stride, int nch, uint32_t (&v)[EB])
+// More than two chunks (long filters with large weights): one wait per chunk.
+template <int EB>
+__device__ __forceinline__ void drain_many(uint32_t a0, uint32_t a1, bool two, int nch, uint32_t stride, uint32_t (&v0)[EB],
+                                        uint32_t (&v1)[EB])
 {
-    constexpr int L = EB < 16 ? 8 : 16;  // columns per TMEM load
-    const int n = NCH > 0 ? NCH : nch;
-#pragma unroll(NCH > 0 ? NCH : 1)
-    for (int c = 0; c < n; ++c) {
-        uint32_t t[EB];
 #pragma unroll
-        for (int b0 = 0; b0 < EB; b0 += L) {
-            if constexpr (L == 16) tmem_ld16(addr + c * stride + b0, *reinterpret_cast<uint32_t(*)[16]>(t + b0));
-            else tmem_ld8(addr + c * stride + b0, *reinterpret_cast<uint32_t(*)[8]>(t + b0));
-        }
+    for (int k = 0; k < EB; ++k) v0[k] = v1[k] = 0;
+#pragma unroll 1
+    for (int c = 0; c < nch; ++c) {
+        uint32_t t0[EB], t1[EB];
+        tmem_load<EB>(a0 + c * stride, t0);
+        if (two) tmem_load<EB>(a1 + c * stride, t1);
         tmem_wait_ld();
 #pragma unroll
-        for (int k = 0; k < EB; ++k) v[k] = c == 0 ? t[k] : v[k] + t[k];
-        tmem_fill<EB>(addr + c * stride);
+        for (int k = 0; k < EB; ++k) {
+            v0[k] += t0[k];
+            v1[k] += t1[k];
+        }
     }
 }
 
-// Compression (Sec. III-A) of G raw chunk sums of one pixel and Q-bit packing.
-// Direct channels use the compact constants dcon = {lam2, kappa | shift << 16}:
-// ((s * kappa + lam2) mod 2^32) >> shift is exact there (see the records).
-template <int BITS, int G>
-__device__ __forceinline__ void win_compress(const uint32_t *s, const uint2 *dcon, const int4 *rec0, const int4 *rec1,
-                                             bool direct, int m_first, uint32_t (&packed)[(G * BITS + 31) / 32])
+template <int EB>
+__device__ __forceinline__ void drain_block(uint32_t a0, uint32_t a1, bool two, int nch, uint32_t stride,
+                                            uint32_t (&v0)[EB], uint32_t (&v1)[EB])
 {
-    int y[G];
-    if (direct) {
+    if (nch <= 2) {
+        uint32_t t0[EB], t1[EB];
+        tmem_load<EB>(a0, v0);
+        if (nch == 2) tmem_load<EB>(a0 + stride, t0);
+        if (two) {
+            tmem_load<EB>(a1, v1);
+            if (nch == 2) tmem_load<EB>(a1 + stride, t1);
+        }
+        tmem_wait_ld();
+        if (nch == 2) {
 #pragma unroll
-        for (int k = 0; k < G; ++k) {
-            const uint2 d = dcon[m_first + k];
-            const uint32_t kap = static_cast<uint32_t>(static_cast<int32_t>(static_cast<int16_t>(d.y & 0xFFFFu)));
-            y[k] = static_cast<int32_t>(s[k] * kap + d.x) >> (d.y >> 16);
+            for (int k = 0; k < EB; ++k) {
+                v0[k] += t0[k];
+                v1[k] += t1[k];  // unused when !two
+            }
         }
     } else {
-#pragma unroll
-        for (int k = 0; k < G; ++k)
-            y[k] = static_cast<int>(compress_slow(s[k], rec0[m_first + k], rec1[m_first + k], (1u << BITS) - 1u));
+        drain_many<EB>(a0, a1, two, nch, stride, v0, v1);
     }
+}
+
+// Q-bit packing of G compressed values (cvt.pack.sat: the clip of Sec. III-A
+// fused with the packing of Sec. IV-A).
+template <int BITS, int G>
+__device__ __forceinline__ void pack_values(const int (&y)[G], uint32_t (&packed)[(G * BITS + 31) / 32])
+{
     constexpr int kPer = 32 / BITS;
     constexpr int kWords = (G * BITS + 31) / 32;
 #pragma unroll
@@ -548,16 +733,35 @@ __device__ __forceinline__ void win_compress(const uint32_t *s, const uint2 *dco
     }
 }
 
+// One block of EB output channels of one strip's pixel: packed Q-bit values,
+// max-pooled over the 2x2 window when POOL (every lane shuffles), stored.
+template <int BITS, int EB, bool POOL>
+__device__ __forceinline__ void store_block(const int (&y)[EB], bool store, int valid, uint8_t *dst)
+{
+    uint32_t pk[(EB * BITS + 31) / 32];
+    pack_values<BITS, EB>(y, pk);
+    if constexpr (POOL) {
+#pragma unroll
+        for (int wd = 0; wd < (EB * BITS + 31) / 32; ++wd) {
+            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 1));
+            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 8));
+        }
+    }
+    if (store) store_packed<BITS, EB>(pk, valid, dst);
+}
+
+// Whether channel m's compression is in the direct form (flags per 16 channels).
+__device__ __forceinline__ bool l_direct(const uint8_t *gdirect, int m) { return gdirect[m >> 4] != 0; }
+
 template <int BITS, int NT, bool POOL>
 __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, uint64_t *acc_full, uint64_t *acc_empty,
                                               const Misc *misc)
 {
-    constexpr int CW = NT / 2;           // columns of this warp
-    constexpr int EB = CW < 32 ? CW : 32;  // columns drained and compressed together
-    constexpr int G = EB < 16 ? EB : 16;   // channels per compression group
+    constexpr int CW = NT / 2;             // columns of this warp
+    constexpr int EB = CW < 8 ? CW : 8;    // columns drained and compressed together (2 strips x 2 chunks in flight)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3, half = (warp - kEpiWarp0) >> 2;
-    const int row = quarter * 32 + lane;  // tile row of the strip: 8 * (output row) + column
+    const int row = quarter * 32 + lane;  // tile row of a strip: 8 * (output row) + column
     const int col0 = half * CW;
     const uint32_t tmem = misc->tmem;
     const int nch = static_cast<int>(misc->nch), nslots = static_cast<int>(misc->nslots);
@@ -565,18 +769,28 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
     const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + col0;
     const int4 *rec0 = reinterpret_cast<const int4 *>(smem + a.off_rec);
     const int4 *rec1 = rec0 + NT;
-    const uint2 *dcon = reinterpret_cast<const uint2 *>(rec1 + NT);
-    const uint8_t *gdirect = reinterpret_cast<const uint8_t *>(dcon + NT);
+    const uint8_t *gdirect = reinterpret_cast<const uint8_t *>(rec1 + NT);
     const int out_row_bytes = a.m * BITS / 8;
-    const int S = a.s;
+    const bool two = a.s == 2;
+    // This warp's channels are fixed: lane l keeps channel col0 + l's direct-form
+    // constants in registers and broadcasts them with shuffles, so the inner loop
+    // touches no shared memory (the tensor cores keep it busy with operand reads).
+    constexpr int LW = CW < 32 ? CW : 32;  // channels per register set
+    uint32_t my_lam2[2], my_kap[2], my_sh[2];
+    bool direct_all = true;
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int m = col0 + (r * 32 < CW ? r * 32 : 0) + lane % LW;
+        const int4 rec = rec0[m];
+        my_lam2[r] = static_cast<uint32_t>(rec.x);
+        my_kap[r] = static_cast<uint32_t>(rec.y);
+        my_sh[r] = static_cast<uint32_t>(rec.z);
+        direct_all = __all_sync(0xffffffffu, l_direct(gdirect, m)) && direct_all;
+    }
+    const uint32_t strip1 = static_cast<uint32_t>(nch) * NT;  // columns from strip 0's buffers to strip 1's
     int *const status = a.status;
 
-    // every buffer this warp reads starts at the pre-load; then all slots are free
-    for (int slot = 0; slot < nslots; ++slot)
-        for (int b = 0; b < S * nch; ++b) tmem_fill<CW>(lane_addr + slot * slot_cols + b * NT);
-    tmem_wait_st();
-    tc_fence_before();
-    __syncwarp();
+    // all slots start free (the MMA warp writes each accumulator's pre-load)
     if (lane == 0)
         for (int slot = 0; slot < nslots; ++slot) mbar_arrive(&acc_empty[slot]);
 
@@ -587,47 +801,61 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
         if (!mbar_wait_warp(&acc_full[slot], (i / nslots) & 1, status)) return;
         tc_fence_after();
         const int oy = g.oy0 + oyr;
-        for (int s = 0; s < S; ++s) {
+        // where strip s's pixel of this lane goes: its output row, or its pooled pixel
+        uint8_t *dst[2];
+        bool store[2];
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
             const int ox = g.ox0 + s * kCols + oxr;
-            const bool pix_ok = oy < a.oh && ox < a.ow;
-            // Fused 2x2/2 max-pool: pooled pixel (oy/2, ox/2) is the window of lanes
-            // L, L^1, L^8, L^9; its top-left lane stores.
-            const bool pool_store = POOL && (row & 9) == 0 && (oy >> 1) < a.pool_oh && (ox >> 1) < a.pool_ow;
-            uint8_t *dst = POOL ? a.y + ((static_cast<long long>(g.img) * a.pool_oh + (oy >> 1)) * a.pool_ow + (ox >> 1)) *
-                                            out_row_bytes
-                                : a.y + ((static_cast<long long>(g.img) * a.oh + oy) * a.ow + ox) * out_row_bytes;
+            if constexpr (POOL) {
+                // pooled pixel (oy/2, ox/2) is the 2x2 window of lanes L, L^1, L^8, L^9; its top-left lane stores
+                store[s] = (row & 9) == 0 && (oy >> 1) < a.pool_oh && (ox >> 1) < a.pool_ow;
+                dst[s] = a.y + ((static_cast<long long>(g.img) * a.pool_oh + (oy >> 1)) * a.pool_ow + (ox >> 1)) *
+                                   out_row_bytes;
+            } else {
+                store[s] = oy < a.oh && ox < a.ow;
+                dst[s] = a.y + ((static_cast<long long>(g.img) * a.oh + oy) * a.ow + ox) * out_row_bytes;
+            }
+            store[s] = store[s] && (s == 0 || two);
+        }
+        const uint32_t base = lane_addr + slot * slot_cols;
+#pragma unroll 1
+        for (int k0 = 0; k0 < CW; k0 += EB) {
+            uint32_t v0[EB], v1[EB];
+            drain_block<EB>(base + k0, base + strip1 + k0, two, nch, NT, v0, v1);
+            if (k0 + EB == CW) {  // the slot's last columns are read: give it back first
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acc_empty[slot]);
+            }
+            const int m0 = col0 + k0;
+            const int valid = a.m - m0;  // same for the whole warp
+            if (valid <= 0) continue;
+            int y0[EB], y1[EB];
+            if (direct_all) {
+                // direct channels: ((s * kappa + lam2) mod 2^32) >> shift is exact (see the records);
+                // the constants of channel col0 + k0 + k sit in lane (k0 + k) % 32 of set (k0 + k) / 32
+                const int set = k0 >= 32 ? 1 : 0;
+                const uint32_t l2 = set ? my_lam2[1] : my_lam2[0], kp = set ? my_kap[1] : my_kap[0];
+                const uint32_t shv = set ? my_sh[1] : my_sh[0];
 #pragma unroll
-            for (int k0 = 0; k0 < CW; k0 += EB) {
-                uint32_t v[EB];
-                const uint32_t src = lane_addr + slot * slot_cols + static_cast<uint32_t>(s * nch) * NT + k0;
-                if (nch == 1) drain<EB, 1>(src, NT, 1, v);
-                else if (nch == 2) drain<EB, 2>(src, NT, 2, v);
-                else drain<EB, 0>(src, NT, nch, v);
-                if (s == S - 1 && k0 + EB == CW) {  // the slot's last columns are read: give it back first
-                    tmem_wait_st();
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&acc_empty[slot]);
+                for (int k = 0; k < EB; ++k) {
+                    const uint32_t lam2 = __shfl_sync(0xffffffffu, l2, (k0 + k) & 31);
+                    const uint32_t kap = __shfl_sync(0xffffffffu, kp, (k0 + k) & 31);
+                    const uint32_t sh = __shfl_sync(0xffffffffu, shv, (k0 + k) & 31);
+                    y0[k] = static_cast<int32_t>(v0[k] * kap + lam2) >> sh;
+                    y1[k] = static_cast<int32_t>(v1[k] * kap + lam2) >> sh;
                 }
+            } else {
 #pragma unroll
-                for (int c = 0; c < EB; c += G) {
-                    const int m0 = col0 + k0 + c;
-                    const int valid = a.m - m0;  // same for the whole warp
-                    if (valid <= 0) continue;
-                    uint32_t pk[(G * BITS + 31) / 32];
-                    win_compress<BITS, G>(v + c, dcon, rec0, rec1, gdirect[m0 >> 4] != 0, m0, pk);
-                    if constexpr (POOL) {
-#pragma unroll
-                        for (int wd = 0; wd < (G * BITS + 31) / 32; ++wd) {  // every lane shuffles
-                            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 1));
-                            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 8));
-                        }
-                        if (pool_store) store_packed<BITS, G>(pk, valid, dst + m0 * BITS / 8);
-                    } else if (pix_ok) {
-                        store_packed<BITS, G>(pk, valid, dst + m0 * BITS / 8);
-                    }
+                for (int k = 0; k < EB; ++k) {
+                    const int4 r0 = rec0[m0 + k], r1 = rec1[m0 + k];
+                    y0[k] = static_cast<int>(compress_slow(v0[k], r0, r1, (1u << BITS) - 1u));
+                    y1[k] = two ? static_cast<int>(compress_slow(v1[k], r0, r1, (1u << BITS) - 1u)) : 0;
                 }
             }
+            store_block<BITS, EB, POOL>(y0, store[0], valid, dst[0] + m0 * BITS / 8);
+            if (two) store_block<BITS, EB, POOL>(y1, store[1], valid, dst[1] + m0 * BITS / 8);
         }
     }
 }
@@ -645,9 +873,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     uint64_t *a_empty = a_full + kMaxStages;
     uint64_t *acc_full = a_empty + kMaxStages;
     uint64_t *acc_empty = acc_full + kMaxSlots;
-    uint64_t *b_ready = acc_empty + kMaxSlots;
-    uint64_t *done = b_ready + 1;
-    Misc *misc = reinterpret_cast<Misc *>(done + 1);
+    uint64_t *done = acc_empty + kMaxSlots;
+    uint64_t *w_full = done + 1;
+    Misc *misc = reinterpret_cast<Misc *>(w_full + 2);  // (one spare barrier slot)
     const int warp = threadIdx.x >> 5;
 
     if (warp == kMmaWarp) {
@@ -662,8 +890,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
                 mbar_init(&acc_full[b], 1);
                 mbar_init(&acc_empty[b], kEpiWarps);
             }
-            mbar_init(b_ready, 1);
             mbar_init(done, 1);
+            mbar_init(w_full, 1);
             fence_mbar_init();
         }
         __syncwarp();
@@ -674,15 +902,24 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     __syncthreads();
     tc_fence_after();
 
+    // The loader starts the copies (filters, then the first windows); the whole
+    // block prepares the filters; then each warp takes its role.
+    LoadState ld{0, 0, static_cast<int>(blockIdx.x), 0u};
+    if (warp == kLoadWarp) {
+        load_filters(a, smem, w_full);
+        load_windows(a, smem, raw_full, raw_empty, ld, a.raw_stages);
+    }
+    prepare_filters<BITS, NT>(a, smem, misc, w_full);
+
     if (warp < kConvWarps) {
         converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
     } else if (warp < kConvWarps + kEpiWarps) {
-        prepare_filters<BITS, NT>(a, smem, misc, b_ready);
         epilogue_role<BITS, NT, POOL>(a, smem, acc_full, acc_empty, misc);
     } else if (warp == kMmaWarp) {
-        mma_role<NT, BITS != 8>(a, smem, a_full, a_empty, acc_full, acc_empty, b_ready, done, misc);
+        mma_role<NT, BITS != 8>(a, smem, a_full, a_empty, acc_full, acc_empty, done, misc);
     } else if (warp == kLoadWarp) {
-        loader_role(a, smem, raw_full, raw_empty);
+        load_windows(a, smem, raw_full, raw_empty, ld, a.total_tiles);
+        load_drain(a, raw_full, w_full, ld);
     }
 
     tc_fence_before();

@@ -178,6 +178,33 @@ __device__ __forceinline__ void mma_f8_ss_warp(uint32_t d_tmem, uint64_t a_desc,
         : "memory");
 }
 
+// The same two MMAs without a "memory" clobber, for issue loops that read their
+// descriptors from shared memory: the compiler may then load the next entries
+// while earlier MMAs are being issued.  The MMAs read their operands through
+// the async proxy; the issuing warp writes no operand memory, and the volatile
+// asm statements (MMAs, commits, barrier waits) keep their relative order.
+__device__ __forceinline__ void mma_f16_ss_warp_nc(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                   uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_f8_ss_warp_nc(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+
 __device__ __forceinline__ void mma_commit_warp(uint64_t *bar)
 {
     asm volatile(

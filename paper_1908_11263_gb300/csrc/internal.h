@@ -93,9 +93,11 @@ struct WinPlan {
     long long total_tiles;
     int full_rows;        // a window spans whole image rows: one bulk copy per tile
     int nch_max;          // exact fp32 chunks the worst-case filters would need
+    int nch_min;          // fewest chunks per strip the kernel considers (1)
     int raw_stages, a_stages;
     uint32_t raw_row_bytes, raw_bytes, b_bytes, chunk_stride, stage_bytes;
-    uint32_t off_b, off_a, off_raw, off_rec, off_thr, off_tap, off_bar, smem_bytes;
+    uint32_t off_b, off_a, off_raw, off_rec, off_thr, off_tap, off_mtab, off_pre, off_wraw, off_bar, smem_bytes;
+    uint32_t wraw_bytes;  // packed filters bulk-copied into shared memory (0: read from global memory)
     size_t param_bytes;   // qconv_hwc_prepare workspace: copies of the filters and constants
     size_t off_pw, off_pbias, off_pkappa, off_plambda, off_pshifts, off_pthr;  // within it
 };

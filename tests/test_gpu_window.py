@@ -18,13 +18,18 @@ def loaded():
     torch.cuda.set_device(0)
 
 
-def centred_lambda(x, wt, bits):
-    """kappa = 1, shift = 0 and a per-channel lambda that centres each channel's accumulators
-    in the output range: every output then depends on the accumulator's last bit."""
+def centred_requant(x, wt, bits):
+    """kappa = 1, a shift matched to the accumulators' spread and a per-channel lambda that
+    centres each channel in the output range: outputs spread over [0, 2^Q - 1] and every
+    output changes with the accumulator at the scale of 2^shift (shift 0 where the spread
+    allows it: then every output depends on the accumulator's last bit)."""
     import oracle
-    acc = oracle.conv_acc(x, wt, (1, 1), (1, 1)).reshape(-1, wt.shape[0])
-    half = 1 << (bits - 1)
-    return (half - np.median(acc, axis=0)).astype(np.int32)
+    acc = oracle.conv_acc(x, wt, (1, 1), (1, 1)).reshape(-1, wt.shape[0]).astype(np.int64)
+    spread = float(np.percentile(acc, 90) - np.percentile(acc, 10))
+    top = (1 << bits) - 1
+    shift = int(max(0, np.ceil(np.log2(max(1.0, spread / (0.8 * top))))))
+    lam = ((top + 1) // 2 * (1 << shift) - np.median(acc, axis=0)).astype(np.int64)
+    return np.clip(lam, -(1 << 31), (1 << 31) - 1).astype(np.int32), shift
 
 
 # (n, h, w, c, m, k): the benchmark layer's shape, C = 64 (K = 576) and a 5x5 window (K = 800)
@@ -50,15 +55,15 @@ def test_chunk_count_from_filters(shape, pattern):
     elif pattern == "alternating":
         wt[..., 0::2] = 127
         wt[..., 1::2] = -128
-    lam = centred_lambda(x, wt, 8)
+    lam, shift = centred_requant(x, wt, 8)
     kappa = np.ones(m, np.int16)
-    want = conv_oracle(x, wt, None, kappa, lam, None, 0, 8, (1, 1), (1, 1))
+    want = conv_oracle(x, wt, None, kappa, lam, None, shift, 8, (1, 1), (1, 1))
     if pattern != "extreme":
         assert len(np.unique(want)) > 32, "outputs nearly constant: the check is weak"
     algos = tc_algos(n, h, w, c, m, k, k, (1, 1), (1, 1), 8)
     assert qnn.ALGO_TC_WINDOW in algos
     for algo in algos:
-        got = conv_gpu(x, wt, None, kappa, lam, None, 0, 8, (1, 1), (1, 1), algo)
+        got = conv_gpu(x, wt, None, kappa, lam, None, shift, 8, (1, 1), (1, 1), algo)
         assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
 
 
@@ -87,7 +92,10 @@ def test_prepared_path(algo, bits, with_bias_and_shifts):
     bias = (taps * top // 4 + rng.integers(-50, 51, size=m)).astype(np.int32) if with_bias_and_shifts else None
     kappa = rng.integers(1, 300, size=m).astype(np.int16)
     shift = {8: 14, 4: 10, 2: 8}[bits]
-    lam = rng.integers(0, (top + 1) << (shift - 1), size=m).astype(np.int32)
+    lam = rng.integers(0, (top + 1) << (shift - 1), size=m).astype(np.int64)
+    if bias is None:  # centre the accumulators through lambda instead (weights average -1/2)
+        lam += (taps * top // 4) * kappa.astype(np.int64)
+    lam = lam.astype(np.int32)
     shifts = rng.integers(shift - 2, shift + 3, size=m).astype(np.uint8) if with_bias_and_shifts else None
     per = 8 // bits
     wd = pack_gpu(wt, bits).view(m, k, k, c // per)

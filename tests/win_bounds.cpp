@@ -20,6 +20,7 @@
 #include <algorithm>
 #include <cstdint>
 #include <cstdio>
+#include <vector>
 
 #include "../paper_1908_11263_gb300/csrc/internal.h"
 
@@ -39,7 +40,7 @@ static int fails = 0;
 // Constants of the kernel (conv_win.cuh).
 static constexpr int kRows = 16, kCols = 8, kConvThreads = 128, kMaxKP = 5, kMaxStages = 4, kMaxSlots = 4;
 static constexpr long long kSmemLimit = 232448;
-static constexpr long long kBarBytes = (4 * kMaxStages + 2 * kMaxSlots + 2) * 8 + 32;
+static constexpr long long kBarBytes = (4 * kMaxStages + 2 * kMaxSlots + 3) * 8 + 32;
 
 // The kernel's reciprocal division: floor(n * m / 2^64), m = ceil(2^64 / d).
 static int fdiv(long long n, unsigned d)
@@ -63,21 +64,62 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
         std::printf("\n");
         return;
     }
-    std::printf(" S=%d %s nt=%d sp=%d wh=%d stages=%d/%d nch_max=%d smem=%u %s\n", p.s, p.fp8 ? "e4m3" : "fp16", p.nt,
-                p.sp, p.wh, p.a_stages, p.raw_stages, p.nch_max, p.smem_bytes, p.full_rows ? "full-rows" : "row-segments");
+    std::printf(" S=%d %s nt=%d sp=%d wh=%d stages=%d/%d nch=%d..%d smem=%u wcopy=%u %s\n", p.s,
+                p.fp8 ? "e4m3" : "fp16", p.nt, p.sp, p.wh, p.a_stages, p.raw_stages, p.nch_min, p.nch_max, p.smem_bytes,
+                p.wraw_bytes, p.full_rows ? "full-rows" : "row-segments");
     const long long cb = static_cast<long long>(c) * bits / 8;
     const int kch = p.fp8 ? 16 : 8, gbytes = kch * bits / 8;  // packed bytes of one K-chunk
-    const int load = bits == 8 ? 8 : (bits == 4 ? 8 : 4);                         // bytes one converter load reads
     CHECK(gbytes == (bits == 8 ? 8 : 16 * bits / 8), "gbytes %d", gbytes);
     const int npos = p.wh * p.sp;
     // shared memory layout
-    const long long rec_bytes = 2LL * p.nt * 16 + p.nt * 8 + p.nt / 16;
+    const long long rec_bytes = 2LL * p.nt * 16 + p.nt / 16;
     CHECK(p.off_b == 0 && p.off_b + p.b_bytes <= p.off_a, "filters");
     CHECK(p.off_a % 128 == 0 && p.off_a + static_cast<long long>(p.a_stages) * p.stage_bytes <= p.off_raw, "stages");
     CHECK(p.off_raw % 128 == 0 && p.off_raw + static_cast<long long>(p.raw_stages) * p.raw_bytes <= p.off_rec, "raw");
     CHECK(p.off_rec % 16 == 0 && p.off_rec + rec_bytes <= p.off_thr, "records");
-    CHECK(p.off_tap + (p.taps + 3LL) * p.nt * 4 <= p.off_bar && p.off_tap % 4 == 0, "tap sums");
+    CHECK(p.off_tap + (p.taps + 3LL) * p.nt * 4 <= p.off_mtab && p.off_tap % 4 == 0, "tap sums");
+    CHECK(p.off_mtab % 8 == 0 && p.off_mtab + 8LL * p.s * p.taps * p.ksteps <= p.off_pre, "MMA table");
+    CHECK(p.off_pre % 128 == 0 && p.off_pre + 4096LL + 32LL * p.nt <= p.off_wraw, "pre-load operands");
+    CHECK(p.off_wraw % 16 == 0 && p.off_wraw + p.wraw_bytes <= p.off_bar, "filter copy");
+    if (p.wraw_bytes) CHECK(p.wraw_bytes == static_cast<long long>(m) * p.taps * cb && p.wraw_bytes % 16 == 0,
+                            "filter copy size");
     CHECK(p.off_bar % 16 == 0 && p.off_bar + kBarBytes <= p.smem_bytes && p.smem_bytes <= kSmemLimit, "barriers");
+    // the MMA issue table the filter preparation writes, for every chunk count the kernel
+    // can take: each entry written once, inside the table, and every (tap, k-step, strip)
+    // issued once into the accumulator of its chunk
+    for (int nch = p.nch_min; nch <= std::max(p.nch_min, p.nch_max); ++nch) {
+        const int ct = (p.taps + nch - 1) / nch, last_len = p.taps - (nch - 1) * ct;
+        if (last_len <= 0) continue;  // the kernel never takes a split with an empty chunk
+        const int nmma = p.s * p.taps * p.ksteps;
+        std::vector<int> seen(nmma, 0), unit(p.taps * p.ksteps * p.s, 0);
+        CHECK(ct * p.ksteps <= 256, "one step pair per preparation thread");
+        for (int et = 0; et < ct * p.ksteps; ++et) {
+            const int jt = et / p.ksteps, kk = et - jt * p.ksteps;
+            const int nj = jt < last_len ? nch : nch - 1;
+            const int before = jt * nch - std::max(0, jt - last_len);
+            int u = p.s * (p.ksteps * before + kk * nj);
+            for (int cc = 0; cc < nj; ++cc) {
+                const int tap = cc * ct + jt;
+                CHECK(tap < p.taps, "table tap");
+                for (int sj = 0; sj < p.s; ++sj, ++u) {
+                    CHECK(u >= 0 && u < nmma, "table index %d", u);
+                    if (u >= 0 && u < nmma) ++seen[u];
+                    ++unit[(tap * p.ksteps + kk) * p.s + sj];
+                    CHECK((sj * nch + cc) * p.nt + p.nt <= 512, "accumulator column");
+                    CHECK(8LL * nmma <= 8LL * p.s * p.taps * p.ksteps, "table size");
+                }
+            }
+        }
+        for (int u = 0; u < nmma; ++u) CHECK(seen[u] == 1, "table entry %d written %d times", u, seen[u]);
+        for (size_t q = 0; q < unit.size(); ++q) CHECK(unit[q] == 1, "MMA unit %zu issued %d times", q, unit[q]);
+    }
+    // MMA table entries: A offset in 16 bits, accumulator column below 512 in the upper 16
+    {
+        const long long a_max = (kh - 1LL) * p.sp + (kw - 1) + (p.ksteps - 1LL) * 2 * (p.chunk_stride / 16) + kCols;
+        CHECK(a_max < 65536, "A offset field");
+        const int cf = std::max(p.nch_min, p.nch_max);
+        CHECK((p.s * cf - 1LL) * p.nt < 512, "accumulator field");
+    }
     CHECK(p.a_stages >= 2 && p.a_stages <= kMaxStages && p.raw_stages >= 2 && p.raw_stages <= kMaxStages, "rings");
     CHECK(p.raw_bytes % 16 == 0 && p.stage_bytes % 16 == 0 && p.chunk_stride % 16 == 0, "16-byte units");
     CHECK(p.chunk_stride >= static_cast<unsigned>(npos) * 16 && p.stage_bytes == p.chunk_stride * p.groups, "planes");
@@ -93,6 +135,11 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
         const int ct = (p.taps + p.nch_max - 1) / p.nch_max;
         CHECK(static_cast<long long>(ct) * p.c_pad * max_prod <= (1LL << 22), "worst-case chunk");
         CHECK((p.nch_max - 1) * ct < p.taps, "empty chunk");
+        // the chunk count the kernel forces whatever the filters: valid by the same bound
+        const int cf = std::max(p.nch_min, p.nch_max), cft = (p.taps + cf - 1) / cf;
+        CHECK(p.nch_min >= 1 && (cf - 1) * cft < p.taps, "forced chunk count %d", cf);
+        CHECK(static_cast<long long>(cft) * p.c_pad * max_prod <= (1LL << 22), "forced chunk bound");
+        CHECK(p.s * cf * p.nt <= 512, "tmem at the forced chunk count");
     }
     CHECK(256 % p.nt == 0 && p.nt >= m, "prep channel per thread");
     // the filter-prep loads: the last K-chunk of the last channel inside the packed filters
@@ -134,22 +181,25 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
                     const bool ok = r >= r0 && r < r1 && px >= c0 && px < c1;
                     const bool inside = iy0 + r >= 0 && iy0 + r < h && ix0 + px >= 0 && ix0 + px < w;
                     CHECK(ok == inside, "staged pixel inside the image");
-                    for (int gq = 0; gq < p.groups; ++gq) {
+                    for (int gq = 0; gq < p.groups; ++gq)
                         CHECK(static_cast<long long>(gq) * p.chunk_stride + pos * 16LL + 16 <= p.stage_bytes, "store");
-                        if (!ok || gq >= c * bits / 8 / gbytes) continue;
-                        const long long src = static_cast<long long>(r - r0) * p.raw_row_bytes + (px + base_col) * cb +
-                                              static_cast<long long>(gq) * gbytes;
-                        CHECK(src >= 0 && src + load <= static_cast<long long>(r1 - r0) * p.raw_row_bytes, "raw load");
-                        // byte q of copied row r stands for global byte row_start + q
-                        const long long row_start =
-                            ((static_cast<long long>(img) * h + iy0 + r) * w + (p.full_rows ? 0 : ix0 + c0)) * cb;
-                        const long long q = src - static_cast<long long>(r - r0) * p.raw_row_bytes;
-                        CHECK(q + load <= seg, "inside the copied span");
-                        const long long want = ((static_cast<long long>(img) * h + iy0 + r) * w + ix0 + px) * cb +
-                                               static_cast<long long>(gq) * gbytes;
-                        CHECK(row_start + q == want, "the pixel's own channels");
-                        CHECK(src % load == 0, "load alignment");
-                    }
+                    // one pixel's packed channels, in 16-byte loads when the pixel is whole
+                    // 16-byte units, else 8-byte ones (a padding position reads the stage's
+                    // first bytes instead)
+                    const int unit = cb % 16 == 0 ? 16 : 8;
+                    CHECK(cb % 8 == 0 && cb <= 64, "pixel bytes");
+                    CHECK(cb <= static_cast<long long>(p.raw_bytes), "padding load");
+                    if (!ok) continue;
+                    const long long src = static_cast<long long>(r - r0) * p.raw_row_bytes + (px + base_col) * cb;
+                    CHECK(src >= 0 && src + cb <= static_cast<long long>(r1 - r0) * p.raw_row_bytes, "raw load");
+                    // byte q of copied row r stands for global byte row_start + q
+                    const long long row_start =
+                        ((static_cast<long long>(img) * h + iy0 + r) * w + (p.full_rows ? 0 : ix0 + c0)) * cb;
+                    const long long q = src - static_cast<long long>(r - r0) * p.raw_row_bytes;
+                    CHECK(q + cb <= seg, "inside the copied span");
+                    const long long want = ((static_cast<long long>(img) * h + iy0 + r) * w + ix0 + px) * cb;
+                    CHECK(row_start + q == want, "the pixel's own channels");
+                    CHECK(src % unit == 0 && p.raw_row_bytes % 16 == 0, "load alignment");
                 }
             // MMA A rows and B rows
             for (int sj = 0; sj < p.s; ++sj)
