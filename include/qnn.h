@@ -89,9 +89,12 @@ typedef struct {
  * the workspace holds the filters re-laid out for the tensor cores and the
  * per-channel compression constants, rewritten by every qconv_hwc() call, so
  * one workspace must not be shared by calls that can run concurrently.  For
- * the window kernel it holds copies of the packed filters, bias, kappa, lambda
- * and shifts, written by qconv_hwc_prepare() only (qconv_hwc() reads the
- * caller's buffers in place and leaves it alone).
+ * the window kernel it holds the image of the kernel's shared-memory operands
+ * that qconv_hwc_prepare() builds once (the filters as the tensor-core B
+ * operand, the per-channel compression records, the exact chunk count and the
+ * MMA issue table); qconv_hwc_run() reads it with two bulk copies per block,
+ * and qconv_hwc() builds the same operands inside its one launch and leaves
+ * the workspace alone.
  */
 qnn_status qconv_hwc_workspace_size(const qnn_conv_desc *d, size_t *bytes);
 
@@ -132,7 +135,8 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
  *
  * qconv_hwc_prepare: writes into `workspace` the filters re-laid out for the
  *   tensor cores and the per-channel constants derived from bias, kappa,
- *   lambda and the shifts (same argument rules as qconv_hwc).  For a
+ *   lambda and the shifts (same argument rules as qconv_hwc); one small
+ *   launch.  The caller's buffers may be freed or changed afterwards.  For a
  *   descriptor that selects the CUDA-core kernel it enqueues nothing.
  * qconv_hwc_run: the convolution itself, reading a workspace prepared for the
  *   same descriptor (any other workspace content gives undefined results).

@@ -189,7 +189,7 @@ qnn_status qconv_hwc_workspace_size(const qnn_conv_desc *d, size_t *bytes)
     if (st != QNN_OK) return st;
     const Choice c = choose(d, s);
     if (c.kernel < 0) return static_cast<qnn_status>(-c.kernel);
-    *bytes = c.kernel == kWindow ? c.wplan.param_bytes : c.kernel == kGeneral ? c.plan.workspace_bytes : 0;
+    *bytes = c.kernel == kWindow ? c.wplan.img_bytes : c.kernel == kGeneral ? c.plan.workspace_bytes : 0;
     return QNN_OK;
 }
 
@@ -238,7 +238,7 @@ qnn_status qconv_hwc_prepare(const qnn_conv_desc *d, const void *w, const int32_
     if (c.kernel == kDirect) return QNN_OK;
     ConvParams p{nullptr, static_cast<const uint8_t *>(w), bias, kappa, lambda, shifts, d->shift, nullptr};
     if (c.kernel == kWindow) {
-        if (!workspace || workspace_bytes < c.wplan.param_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
+        if (!workspace || workspace_bytes < c.wplan.img_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
         return from_cuda(prepare_conv_win(c.wplan, s, p, workspace, static_cast<cudaStream_t>(stream)));
     }
     st = check_workspace(plan, workspace, workspace_bytes);
@@ -258,11 +258,11 @@ qnn_status qconv_hwc_run(const qnn_conv_desc *d, const void *x, void *y, const v
     if (c.kernel < 0) return static_cast<qnn_status>(-c.kernel);
     if (c.kernel == kDirect) return QNN_EUNSUPPORTED;
     if (c.kernel == kWindow) {
-        if (!workspace || workspace_bytes < c.wplan.param_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
-        ConvParams p = win_prepared_params(c.wplan, workspace);
+        if (!workspace || workspace_bytes < c.wplan.img_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
+        ConvParams p{};
         p.x = static_cast<const uint8_t *>(x);
         p.y = static_cast<uint8_t *>(y);
-        return from_cuda(launch_conv_win(c.wplan, s, p, static_cast<cudaStream_t>(stream)));
+        return from_cuda(launch_conv_win(c.wplan, s, p, static_cast<cudaStream_t>(stream), workspace));
     }
     st = check_workspace(c.plan, workspace, workspace_bytes);
     if (st != QNN_OK) return st;

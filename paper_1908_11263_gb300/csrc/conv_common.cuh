@@ -246,7 +246,8 @@ __device__ __forceinline__ void store_packed(const uint32_t (&packed)[(G * BITS 
         if (kBytes == 16) *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
         else if (kBytes == 8) *reinterpret_cast<uint2 *>(dst) = make_uint2(packed[0], packed[kWords > 1 ? 1 : 0]);
         else if (kBytes == 4) *reinterpret_cast<uint32_t *>(dst) = packed[0];
-        else *reinterpret_cast<uint16_t *>(dst) = static_cast<uint16_t>(packed[0]);
+        else if (kBytes == 2) *reinterpret_cast<uint16_t *>(dst) = static_cast<uint16_t>(packed[0]);
+        else *dst = static_cast<uint8_t>(packed[0]);
     } else {
         const int nbytes = min(valid, G) * BITS / 8;
 #pragma unroll

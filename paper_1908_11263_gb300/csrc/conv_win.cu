@@ -150,24 +150,19 @@ WinPlan plan_conv_win(const ConvShape &s)
         p.b_bytes = b_bytes;
         p.chunk_stride = chunk_stride;
         p.stage_bytes = stage_bytes;
-        // prepared workspace: the packed filters, bias, kappa, lambda and shifts
-        const size_t wbytes = static_cast<size_t>(s.m) * p.taps * static_cast<size_t>(cb);
-        p.off_pw = 0;
-        p.off_pbias = round_up_sz(wbytes, 256);
-        p.off_pkappa = round_up_sz(p.off_pbias + 4 * static_cast<size_t>(s.m), 256);
-        p.off_plambda = round_up_sz(p.off_pkappa + 2 * static_cast<size_t>(s.m), 256);
-        p.off_pshifts = round_up_sz(p.off_plambda + 4 * static_cast<size_t>(s.m), 256);
-        p.off_pthr = round_up_sz(p.off_pshifts + static_cast<size_t>(s.m), 256);
-        p.param_bytes = p.off_pthr;
+        // prepared workspace: the image of B and the tail
+        p.tail_bytes = p.off_pre + 4096u + static_cast<uint32_t>(p.nt) * 32u - p.off_rec;
+        p.img_bytes = round_up_sz(static_cast<size_t>(b_bytes) + p.tail_bytes, 256);
         p.ok = true;
         return p;
     }
     return p;
 }
 
-cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, cudaStream_t st)
+namespace {
+
+win::WinArgs win_args(const WinPlan &plan, const ConvShape &s, const ConvParams &p)
 {
-    if (s.n == 0) return cudaSuccess;
     win::WinArgs a{};
     a.x = p.x;
     a.y = p.y;
@@ -218,10 +213,15 @@ cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvP
     a.pool = s.pool;
     a.pool_oh = s.oh / 2;
     a.pool_ow = s.ow / 2;
+    a.b_bytes = plan.b_bytes;
+    a.tail_bytes = plan.tail_bytes;
     a.status = device_status_ptr();
+    return a;
+}
+
+cudaError_t launch_win(const WinPlan &plan, const ConvShape &s, const win::WinArgs &a, int grid, cudaStream_t st)
+{
     if (!a.status) return cudaErrorInvalidSymbol;
-    const long long sms = device_sm_count();
-    const int grid = static_cast<int>(std::min<long long>(plan.total_tiles, sms));
     switch (s.bits) {
         case 8: return launch_win_bits<8>(a, plan.nt, grid, plan.smem_bytes, st);
         case 4: return launch_win_bits<4>(a, plan.nt, grid, plan.smem_bytes, st);
@@ -229,40 +229,28 @@ cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvP
     }
 }
 
+}  // namespace
+
+cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, cudaStream_t st,
+                            const void *img)
+{
+    if (s.n == 0) return cudaSuccess;
+    win::WinArgs a = win_args(plan, s, p);
+    if (img) {
+        a.img = static_cast<const uint8_t *>(img);
+        a.wraw_bytes = 0;  // no filter copy: the image replaces it
+    }
+    const long long sms = device_sm_count();
+    const int grid = static_cast<int>(std::min<long long>(plan.total_tiles, sms));
+    return launch_win(plan, s, a, grid, st);
+}
+
 cudaError_t prepare_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
                              cudaStream_t st)
 {
-    uint8_t *ws = static_cast<uint8_t *>(workspace);
-    const size_t wbytes = static_cast<size_t>(s.m) * plan.taps * (static_cast<size_t>(s.c) * s.bits / 8);
-    cudaError_t e = cudaMemcpyAsync(ws + plan.off_pw, p.w, wbytes, cudaMemcpyDeviceToDevice, st);
-    if (e == cudaSuccess)
-        e = p.bias ? cudaMemcpyAsync(ws + plan.off_pbias, p.bias, 4 * static_cast<size_t>(s.m),
-                                     cudaMemcpyDeviceToDevice, st)
-                   : cudaMemsetAsync(ws + plan.off_pbias, 0, 4 * static_cast<size_t>(s.m), st);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(ws + plan.off_pkappa, p.kappa, 2 * static_cast<size_t>(s.m), cudaMemcpyDeviceToDevice, st);
-    if (e == cudaSuccess)
-        e = cudaMemcpyAsync(ws + plan.off_plambda, p.lambda, 4 * static_cast<size_t>(s.m), cudaMemcpyDeviceToDevice,
-                            st);
-    if (e == cudaSuccess)
-        e = p.shifts ? cudaMemcpyAsync(ws + plan.off_pshifts, p.shifts, static_cast<size_t>(s.m),
-                                       cudaMemcpyDeviceToDevice, st)
-                     : cudaMemsetAsync(ws + plan.off_pshifts, p.shift, static_cast<size_t>(s.m), st);
-    return e;
-}
-
-ConvParams win_prepared_params(const WinPlan &plan, const void *workspace)
-{
-    const uint8_t *ws = static_cast<const uint8_t *>(workspace);
-    ConvParams p{};
-    p.w = ws + plan.off_pw;
-    p.bias = reinterpret_cast<const int32_t *>(ws + plan.off_pbias);
-    p.kappa = reinterpret_cast<const int16_t *>(ws + plan.off_pkappa);
-    p.lambda = reinterpret_cast<const int32_t *>(ws + plan.off_plambda);
-    p.shifts = ws + plan.off_pshifts;
-    p.shift = 0;
-    p.thresholds = nullptr;
-    return p;
+    win::WinArgs a = win_args(plan, s, p);
+    a.img_out = static_cast<uint8_t *>(workspace);
+    return launch_win(plan, s, a, 1, st);
 }
 
 }  // namespace qnn

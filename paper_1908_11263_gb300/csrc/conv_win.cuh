@@ -58,6 +58,11 @@ constexpr int kConvWarps = 4, kEpiWarps = 8;
 constexpr int kEpiWarp0 = 4, kMmaWarp = 12, kLoadWarp = 13;
 constexpr int kWarps = 14;
 constexpr int kThreads = kWarps * 32;
+// the filter preparation runs on the epilogue warps and the MMA warp (the
+// warps that use its results), synchronised by named barrier 1; the
+// converters and the loader start on the first windows meanwhile
+constexpr int kPrepWarp0 = kEpiWarp0;
+constexpr int kPrepThreads = (kMmaWarp + 1 - kPrepWarp0) * 32;
 constexpr int kRows = 16, kCols = 8;  // output rows and columns of one strip
 constexpr int kMaxTaps = 64;
 constexpr int kMaxSlots = 4;          // accumulator slots in TMEM
@@ -70,12 +75,13 @@ constexpr int kSmemLimit = 232448;    // 227 KB opt-in dynamic shared memory per
 // the MMAs per tile.
 struct Misc {
     uint32_t tmem;
-    uint32_t nch;
+    uint32_t nch;  // accumulators per strip: exact chunks x K-split
     uint32_t nslots;
     uint32_t slot_cols;
     uint32_t mask;
     uint32_t nmma;  // MMAs per tile (entries of the issue table)
-    uint32_t pad[2];
+    uint32_t kx;    // K-split: the k-steps of a tap alternate between kx accumulators
+    uint32_t pad;
 };
 
 struct WinArgs {
@@ -100,6 +106,13 @@ struct WinArgs {
     uint32_t off_wraw, wraw_bytes;  // packed filters copied into shared memory (0 bytes: read from global)
     uint32_t off_mtab;              // the MMA issue table (S * taps * ksteps entries of 8 bytes)
     uint32_t off_pre;               // operands of the pre-load MMA (A 4 KB, then B 2 * NT * 16 bytes)
+    // The prepared image: B ([off_b, off_b + b_bytes)) followed by the tail
+    // [off_rec, off_rec + tail_bytes) (records, thresholds, tap sums with the
+    // chunk count, MMA table, pre-load operands).  img: read it instead of
+    // preparing the filters; img_out: prepare, write it and stop (one block).
+    const uint8_t *img;
+    uint8_t *img_out;
+    uint32_t b_bytes, tail_bytes;
     int pool, pool_oh, pool_ow;
     int *status;
 };
@@ -331,10 +344,13 @@ __device__ __forceinline__ void mma_nc(uint32_t d, uint64_t ad, uint64_t bd, uin
 }
 
 // One tile's MMAs with every offset known at compile time (one exact chunk,
-// KH x KW taps, KS k-steps per tap, S strips): a descriptor is its template's
-// low word plus an offset (a start address field that cannot carry out of its
-// 14 bits), so each MMA costs an addition or two and the issue.
-template <int KH, int KW, int KS, int S, int NT, bool F8>
+// KH x KW taps, KS k-steps per tap, S strips, k-step kk of a tap into the
+// strip's accumulator kk % KX): a descriptor is its template's low word plus
+// an offset (a start address field that cannot carry out of its 14 bits), so
+// each MMA costs an addition or two and the issue.  Consecutive MMAs go to
+// S * KX different accumulators: an MMA into the accumulator the previous one
+// wrote waits for it, so one chain runs at about half the tensor pipe's rate.
+template <int KH, int KW, int KS, int S, int NT, bool F8, int KX>
 __device__ __forceinline__ void issue_fixed(uint32_t d0, uint32_t alo, uint32_t ahi, uint32_t blo, uint32_t bhi,
                                             uint32_t idesc, int sp, uint32_t kstep_a)
 {
@@ -349,7 +365,8 @@ __device__ __forceinline__ void issue_fixed(uint32_t d0, uint32_t alo, uint32_t 
                 const uint64_t bd = desc_of(blo + static_cast<uint32_t>(((i * KW + j) * 2 * KS + 2 * kk) * NT), bhi);
 #pragma unroll
                 for (int s = 0; s < S; ++s)
-                    mma_nc<F8>(d0 + s * NT, desc_of(arow + j + kk * kstep_a + s * kCols, ahi), bd, idesc);
+                    mma_nc<F8>(d0 + (s * KX + kk % KX) * NT, desc_of(arow + j + kk * kstep_a + s * kCols, ahi), bd,
+                               idesc);
             }
     }
 }
@@ -373,12 +390,13 @@ __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64
     const uint64_t pre_a = smem_desc(0, 2048, 128) + pre16;
     const uint64_t pre_b = smem_desc(0, NT * 16, 128) + pre16 + 256;
     const int nacc = a.s * nch;
+    const int kx = static_cast<int>(misc->kx);
     // the issue order (built by the filter preparation): one 8-byte entry per MMA,
     // {A offset in 16-byte units | accumulator column << 16, B offset}
     const uint2 *tab = reinterpret_cast<const uint2 *>(smem + a.off_mtab);
     const int nu = static_cast<int>(misc->nmma);
     // the common shapes with one exact chunk issue from unrolled code
-    const int fixed = nch != 1 ? 0
+    const int fixed = nch != kx ? 0
                       : (a.kh == 3 && a.kw == 3 && a.ksteps == 2 && a.s == 2) ? 1
                       : (a.kh == 3 && a.kw == 3 && a.ksteps == 1 && a.s == 2) ? 2
                       : (a.kh == 5 && a.kw == 5 && a.ksteps == 2 && a.s == 2) ? 3
@@ -397,12 +415,16 @@ __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64
         for (int b = 0; b < nacc; ++b) mma_f16_ss_warp_nc(d0 + b * NT, pre_a, pre_b, idesc, 0u);
         const uint32_t alo = static_cast<uint32_t>(abase), ahi = static_cast<uint32_t>(abase >> 32);
         const uint32_t blo = static_cast<uint32_t>(bbase), bhi = static_cast<uint32_t>(bbase >> 32);
-        switch (fixed) {
-            case 1: issue_fixed<3, 3, 2, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
-            case 2: issue_fixed<3, 3, 1, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
-            case 3: issue_fixed<5, 5, 2, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
-            case 4: issue_fixed<5, 5, 2, 1, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
-            case 5: issue_fixed<3, 3, 4, 2, NT, F8>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+        switch (fixed * 2 + (kx == 2 ? 1 : 0)) {
+            case 2: issue_fixed<3, 3, 2, 2, NT, F8, 1>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 3: issue_fixed<3, 3, 2, 2, NT, F8, 2>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 4: issue_fixed<3, 3, 1, 2, NT, F8, 1>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 6: issue_fixed<5, 5, 2, 2, NT, F8, 1>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 7: issue_fixed<5, 5, 2, 2, NT, F8, 2>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 8: issue_fixed<5, 5, 2, 1, NT, F8, 1>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 9: issue_fixed<5, 5, 2, 1, NT, F8, 2>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 10: issue_fixed<3, 3, 4, 2, NT, F8, 1>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
+            case 11: issue_fixed<3, 3, 4, 2, NT, F8, 2>(d0, alo, ahi, blo, bhi, idesc, a.sp, kstep_a); break;
             default:
 #pragma unroll 4
                 for (int u = 0; u < nu; ++u) {
@@ -418,27 +440,30 @@ __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64
     mbar_wait_warp(done, 0, status);
 }
 
-// ---------------------------------------------------------------- filter preparation (the whole block)
+// ---------------------------------------------------------------- filter preparation (warps 4-12)
+
+__device__ __forceinline__ void prep_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kPrepThreads) : "memory"); }
 
 // One K-chunk of one output channel's filter at one tap, from its packed
 // bytes (8, or 4 at INT-2, in v): the staged B row (8 fp16 or 16 e4m3 values
 // in the converter's channel order) and the sums the compression constants and
 // the chunk count need.
 template <int BITS>
-__device__ __forceinline__ uint4 filter_chunk(uint2 v, int &sum, int &pos, int &neg, int &abs)
+__device__ __forceinline__ uint4 filter_chunk(uint2 v, int &pos, int &neg, int &abs)
 {
-    if (BITS == 8) {
-        // byte sums by 4-way signed dot products with ones: the weights, and their negative parts
+    if constexpr (BITS == 8) {
+        // byte sums by 4-way signed dot products with ones: all weights, and the
+        // negative ones (prmt with a sign-replicating selector gives 0xFF in
+        // every negative byte)
         const int all = __dp4a(static_cast<int>(v.x), 0x01010101, __dp4a(static_cast<int>(v.y), 0x01010101, 0));
-        const int ng = __dp4a(static_cast<int>(__vmins4(v.x, 0u)), 0x01010101,
-                              __dp4a(static_cast<int>(__vmins4(v.y, 0u)), 0x01010101, 0));
-        sum += all;
+        const uint32_t nx = v.x & prmt(v.x, 0u, 0xBA98u), ny = v.y & prmt(v.y, 0u, 0xBA98u);
+        const int ng = __dp4a(static_cast<int>(nx), 0x01010101, __dp4a(static_cast<int>(ny), 0x01010101, 0));
         neg += ng;
         pos += all - ng;
         abs += all - 2 * ng;
         // byte b ^ 0x80 is the weight plus 128 as an unsigned byte: the activation encoding gives the weight
         return cvt_u8x8(make_uint2(v.x ^ 0x80808080u, v.y ^ 0x80808080u));
-    }
+    } else {
     uint8_t e[16];
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
@@ -446,7 +471,6 @@ __device__ __forceinline__ uint4 filter_chunk(uint2 v, int &sum, int &pos, int &
         const uint32_t word = k / per == 0 ? v.x : v.y;
         const int f = (word >> ((k % per) * BITS)) & ((1 << BITS) - 1);
         const int wv = f >= (1 << (BITS - 1)) ? f - (1 << BITS) : f;
-        sum += wv;
         pos += max(wv, 0);
         neg += min(wv, 0);
         abs += wv < 0 ? -wv : wv;
@@ -460,40 +484,39 @@ __device__ __forceinline__ uint4 filter_chunk(uint2 v, int &sum, int &pos, int &
     r.z = e[8] | e[9] << 8 | e[10] << 16 | static_cast<uint32_t>(e[11]) << 24;
     r.w = e[12] | e[13] << 8 | e[14] << 16 | static_cast<uint32_t>(e[15]) << 24;
     return r;
+    }
 }
 
-// The B operand ([tap][K-chunk][NT rows][16 B]), the chunk count, the
-// per-channel compression records (rec0 = {lam2, kappa, shift, mode},
-// rec1 = {beta, ulo, uhi, lambda}, as in the tensor-core prep kernel, with
-// acc + bias = s + beta for the raw chunk sum s) and the accumulator slots.
+// What the MMA warp needs, made by warps 4-12 together: the B operand
+// ([tap][K-chunk][NT rows][16 B]), the per-(channel, tap) absolute sums and
+// the chunk count they allow, the MMA issue table, the pre-load operands and
+// the slot layout.  The per-channel sums of positive and negative weights
+// stay in shared memory for the compression records.
 template <int BITS, int NT>
 __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem, Misc *misc, uint64_t *w_full)
 {
     constexpr int kGroupBytes = BITS == 8 ? 8 : 16 * BITS / 8;
     constexpr int kMaxX = BITS == 8 ? 128 : (1 << BITS) - 1;  // largest |staged activation|
-    constexpr int kItemThreads = kThreads / NT * NT;            // threads with a filter item: a multiple of NT
-    const int et = threadIdx.x;
+    constexpr int kBatch = 2;                                   // items per thread whose loads go out together
+    const int et = threadIdx.x - kPrepWarp0 * 32;
     int *tapabs = reinterpret_cast<int *>(smem + a.off_tap);    // [taps][NT]
-    int *sums = tapabs + a.taps * NT;                           // [3][NT]: sum, positive part, negative part
-    for (int i = et; i < 3 * NT; i += kThreads) sums[i] = 0;
+    int *sums = tapabs + a.taps * NT;                           // [2][NT]: positive part, negative part
+    for (int i = et; i < 2 * NT; i += kPrepThreads) sums[i] = 0;
     if (et == 0) misc->mask = ~0u;
-    __syncthreads();
-    // item i: channel n = i % NT (fixed per thread: kItemThreads is a multiple of NT), tap i / NT.
-    // Every load of a batch of two items goes out before any of them is used.
+    prep_sync();
+    // item i: channel n = i % NT, tap i / NT; thread et takes items et, et + kPrepThreads, ...
     const int cgroups = a.c * BITS / 8 / kGroupBytes;
-    int sum = 0, pos = 0, neg = 0;
-    const int n = et % NT;
     const int items = a.taps * NT;
     const long long wrow = static_cast<long long>(a.c) * BITS / 8;  // packed bytes of one tap of one filter
     // the packed filters: the loader's shared-memory copy, or global memory
     const bool copied = a.wraw_bytes != 0;
     if (copied) mbar_wait_warp(w_full, 0, a.status);
     const uint8_t *wsrc = copied ? smem + a.off_wraw : a.w;
-    for (int i0 = et; et < kItemThreads && i0 < items; i0 += 2 * kItemThreads) {
-        uint2 raw[2][8];
+    for (int i0 = et; i0 < items; i0 += kBatch * kPrepThreads) {
+        uint2 raw[kBatch][8];
 #pragma unroll
-        for (int b = 0; b < 2; ++b) {
-            const int i = i0 + b * kItemThreads;
+        for (int b = 0; b < kBatch; ++b) {
+            const int i = i0 + b * kPrepThreads, n = i % NT;
             const uint8_t *src = wsrc + (static_cast<long long>(n) * a.taps + i / NT) * wrow;
 #pragma unroll
             for (int gq = 0; gq < 8; ++gq) {
@@ -508,28 +531,41 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
             }
         }
 #pragma unroll
-        for (int b = 0; b < 2; ++b) {
-            const int i = i0 + b * kItemThreads;
+        for (int b = 0; b < kBatch; ++b) {
+            const int i = i0 + b * kPrepThreads;
             if (i >= items) break;
-            const int tap = i / NT;
-            int abs = 0;
+            const int n = i % NT, tap = i / NT;
+            int pos = 0, neg = 0, abs = 0;
 #pragma unroll
             for (int gq = 0; gq < 8; ++gq) {
                 if (gq >= a.groups) break;
                 // K-chunks past the channel count (and filters past m) stage +0
-                const uint4 v = (n < a.m && gq < cgroups) ? filter_chunk<BITS>(raw[b][gq], sum, pos, neg, abs)
+                const uint4 v = (n < a.m && gq < cgroups) ? filter_chunk<BITS>(raw[b][gq], pos, neg, abs)
                                                          : make_uint4(0u, 0u, 0u, 0u);
                 *reinterpret_cast<uint4 *>(smem + a.off_b + ((tap * a.groups + gq) * NT + n) * 16) = v;
             }
             tapabs[tap * NT + n] = abs;
+            if (n < a.m) {
+                atomicAdd(&sums[n], pos);
+                atomicAdd(&sums[NT + n], neg);
+            }
         }
     }
-    if (et < kItemThreads && items > et) {  // this thread saw channel n
-        atomicAdd(&sums[n], sum);
-        atomicAdd(&sums[NT + n], pos);
-        atomicAdd(&sums[2 * NT + n], neg);
+    // Operands of the pre-load MMA (K-major, 8-row core matrices 128 bytes apart,
+    // the second K-chunk 16 rows further): A rows {2048, 0, ...}, B rows {6144, 0, ...},
+    // so every accumulator element becomes 2048 * 6144 = 1.5 * 2^23.
+    {
+        uint32_t *pre = reinterpret_cast<uint32_t *>(smem + a.off_pre);
+        const int aw = 128 * 2 * 4, bw = NT * 2 * 4;  // 32-bit words: A (128 rows, 2 chunks), B (NT rows, 2 chunks)
+        for (int i = et; i < aw + bw; i += kPrepThreads) {
+            const bool is_a = i < aw;
+            const int j = is_a ? i : i - aw;       // word within the operand
+            const int rows = is_a ? 128 : NT;
+            const bool first = j < rows * 4 && (j & 3) == 0;  // chunk 0, element 0 of a row
+            pre[i] = first ? (is_a ? 0x6800u : 0x6E00u) : 0u;  // fp16 2048, 6144
+        }
     }
-    __syncthreads();
+    prep_sync();
     // Chunk counts c in [nch_min, c_force] whose even tap split has no empty
     // chunk and keeps every chunk of every channel exact; c_force = max(nch_min,
     // nch_max) holds by the planner's worst-case bound whatever the filters.
@@ -550,52 +586,14 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
         okmask |= 1u << c_force;
         atomicAnd(&misc->mask, okmask);
     }
-    __syncthreads();
+    prep_sync();
     const int nch = __ffs(static_cast<int>(misc->mask)) - 1;
-    // per-channel records
-    int4 *rec0 = reinterpret_cast<int4 *>(smem + a.off_rec);
-    int4 *rec1 = rec0 + NT;
-    if (et < NT) {
-        const int o = et;
-        const long long off = BITS == 8 ? -128 : 0;  // staged activation = x + off
-        const int s_w = sums[o];
-        int4 r0 = make_int4(0, 0, 0, kModeDirect), r1 = make_int4(0, 0, 0, 0);
-        if (a.thr) {
-            // staircase: the epilogue compares acc = s + beta with the thresholds
-            const uint32_t beta = 0u - static_cast<uint32_t>(off * s_w) - static_cast<uint32_t>(nch) * kMagic;
-            int32_t *ts = reinterpret_cast<int32_t *>(smem + a.off_thr) + o * kThrStride;
-            for (int k = 0; k < kThrStride; ++k)
-                ts[k] = (o < a.m && k < (1 << BITS) - 1) ? a.thr[static_cast<long long>(o) * ((1 << BITS) - 1) + k]
-                                                        : INT32_MAX;
-            r0 = make_int4(static_cast<int>(a.off_thr) + o * 4 * kThrStride, 0, 0, kModeThreshold);
-            r1 = make_int4(static_cast<int32_t>(beta), 0, 0, 0);
-        } else if (o < a.m) {
-            const int32_t b = a.bias ? a.bias[o] : 0;
-            const uint32_t beta = static_cast<uint32_t>(b) - static_cast<uint32_t>(off * s_w) -
-                                  static_cast<uint32_t>(nch) * kMagic;
-            const int32_t kap = a.kappa[o], lam = a.lambda[o], sh = a.shifts ? a.shifts[o] : a.shift;
-            const long long top = (1 << BITS) - 1;
-            // every accumulator of this channel lies in [top * neg, top * pos]
-            const long long u0 = top * sums[2 * NT + o] + b, u1 = top * sums[NT + o] + b;
-            const bool direct = in_i32(u0 * kap + lam) && in_i32(u1 * kap + lam);
-            long long ulo = 0, uhi = 0;
-            const bool clamp = !direct && saturation_bounds(kap, lam, sh, top, &ulo, &uhi);
-            const int mode = direct ? kModeDirect : clamp ? kModeClamp : kModeWide;
-            const uint32_t lam2 = beta * static_cast<uint32_t>(kap) + static_cast<uint32_t>(lam);
-            r0 = make_int4(static_cast<int32_t>(lam2), kap, sh, mode);
-            r1 = make_int4(static_cast<int32_t>(beta), static_cast<int32_t>(ulo), static_cast<int32_t>(uhi), lam);
-        }
-        rec0[o] = r0;
-        rec1[o] = r1;
-    }
-    __syncthreads();
-    // one "all direct" flag per 16-channel group
-    uint8_t *gd = reinterpret_cast<uint8_t *>(rec1 + NT);
-    if (et < NT / 16) {
-        int all = 1;
-        for (int k = 0; k < 16; ++k) all &= rec0[et * 16 + k].w == kModeDirect;
-        gd[et] = static_cast<uint8_t>(all);
-    }
+    // K-split: a tile with a single accumulator (one strip, one chunk) and an
+    // even k-step count alternates the k-steps of a tap between two
+    // accumulators (each sums a subset of the chunk's products, so each is
+    // exact where the chunk is), so that consecutive MMAs do not wait on each
+    // other; the epilogue adds all nch * kx accumulators of a strip
+    const int kx = (a.s * nch == 1 && a.ksteps % 2 == 0 && 2 * NT <= 256) ? 2 : 1;
     // The MMA issue order, one 8-byte entry per MMA: {A offset (16-byte units
     // within a stage) | accumulator column << 16, B offset}.  The accumulators
     // (chunk c, strip s) are independent and consecutive MMAs go to different
@@ -615,40 +613,129 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
             const int tap = c * ct + jt, ti = tap / a.kw, tj = tap - ti * a.kw;
             for (int s = 0; s < a.s; ++s, ++u)
                 tab[u] = make_uint2((static_cast<uint32_t>(ti * a.sp + tj) + kk * kstep_a + s * kCols) |
-                                        (static_cast<uint32_t>(s * nch + c) * NT << 16),
+                                        (static_cast<uint32_t>((s * nch + c) * kx + kk % kx) * NT << 16),
                                     static_cast<uint32_t>(tap * a.groups) * NT + kk * kstep_b);
         }
     }
-    // Operands of the pre-load MMA (K-major, 8-row core matrices 128 bytes apart,
-    // the second K-chunk 16 rows further): A rows {2048, 0, ...}, B rows {6144, 0, ...},
-    // so every accumulator element becomes 2048 * 6144 = 1.5 * 2^23.
-    {
-        uint32_t *pre = reinterpret_cast<uint32_t *>(smem + a.off_pre);
-        const int aw = 128 * 2 * 4, bw = NT * 2 * 4;  // 32-bit words: A (128 rows, 2 chunks), B (NT rows, 2 chunks)
-        for (int i = et; i < aw + bw; i += kThreads) {
-            const bool is_a = i < aw;
-            const int j = is_a ? i : i - aw;       // word within the operand
-            const int rows = is_a ? 128 : NT;
-            const bool first = j < rows * 4 && (j & 3) == 0;  // chunk 0, element 0 of a row
-            pre[i] = first ? (is_a ? 0x6800u : 0x6E00u) : 0u;  // fp16 2048, 6144
-        }
-    }
-    // B and the pre-load operands were written through the generic proxy; the
-    // tensor cores read them through the async proxy
-    fence_proxy_async_smem();
-    __syncthreads();
     if (et == 0) {
-        const uint32_t cols = static_cast<uint32_t>(a.s * nch * NT);
-        misc->nch = static_cast<uint32_t>(nch);
+        const uint32_t cols = static_cast<uint32_t>(a.s * nch * kx * NT);
+        misc->nch = static_cast<uint32_t>(nch * kx);
+        misc->kx = static_cast<uint32_t>(kx);
+        // the tap area's spare row carries both into a prepared image
+        tapabs[(a.taps + 2) * NT] = nch * kx;
+        tapabs[(a.taps + 2) * NT + 1] = kx;
         misc->slot_cols = cols;
         misc->nslots = min(static_cast<uint32_t>(kMaxSlots), 512u / cols);
         misc->nmma = static_cast<uint32_t>(a.s * a.taps * a.ksteps);
     }
-    // the roles start after this barrier: B, the records, the table and the
-    // slot layout are complete
+    // B and the pre-load operands were written through the generic proxy; the
+    // tensor cores read them through the async proxy
+    fence_proxy_async_smem();
+    // the MMA warp starts after this barrier: B, the table and the slot layout are complete
     tc_fence_before();
-    __syncthreads();
+    prep_sync();
     tc_fence_after();
+}
+
+// The per-channel compression records (rec0 = {lam2, kappa, shift, mode},
+// rec1 = {beta, ulo, uhi, lambda}, as in the tensor-core prep kernel, with
+// acc + bias = s + beta for the raw chunk sum s) and the "all direct" flag of
+// every 16 channels, made by the epilogue warps while the first tile's MMAs
+// run (named barrier 2).
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 2, %0;" ::"n"(kEpiWarps * 32) : "memory"); }
+
+template <int BITS, int NT>
+__device__ __forceinline__ void prepare_records(const WinArgs &a, uint8_t *smem, const Misc *misc)
+{
+    const int et = threadIdx.x - kEpiWarp0 * 32;
+    const int *sums = reinterpret_cast<const int *>(smem + a.off_tap) + a.taps * NT;
+    const int nch = static_cast<int>(misc->nch);
+    int4 *rec0 = reinterpret_cast<int4 *>(smem + a.off_rec);
+    int4 *rec1 = rec0 + NT;
+    if (et < NT) {
+        const int o = et;
+        const long long off = BITS == 8 ? -128 : 0;  // staged activation = x + off
+        const int s_w = sums[o] + sums[NT + o];
+        int4 r0 = make_int4(0, 0, 0, kModeDirect), r1 = make_int4(0, 0, 0, 0);
+        if (a.thr) {
+            // staircase: the epilogue compares acc = s + beta with the thresholds
+            const uint32_t beta = 0u - static_cast<uint32_t>(off * s_w) - static_cast<uint32_t>(nch) * kMagic;
+            int32_t *ts = reinterpret_cast<int32_t *>(smem + a.off_thr) + o * kThrStride;
+            for (int k = 0; k < kThrStride; ++k)
+                ts[k] = (o < a.m && k < (1 << BITS) - 1) ? a.thr[static_cast<long long>(o) * ((1 << BITS) - 1) + k]
+                                                        : INT32_MAX;
+            r0 = make_int4(static_cast<int>(a.off_thr) + o * 4 * kThrStride, 0, 0, kModeThreshold);
+            r1 = make_int4(static_cast<int32_t>(beta), 0, 0, 0);
+        } else if (o < a.m) {
+            const int32_t b = a.bias ? a.bias[o] : 0;
+            const uint32_t beta = static_cast<uint32_t>(b) - static_cast<uint32_t>(off * s_w) -
+                                  static_cast<uint32_t>(nch) * kMagic;
+            const int32_t kap = a.kappa[o], lam = a.lambda[o], sh = a.shifts ? a.shifts[o] : a.shift;
+            const long long top = (1 << BITS) - 1;
+            // every accumulator of this channel lies in [top * neg, top * pos]
+            const long long u0 = top * sums[NT + o] + b, u1 = top * sums[o] + b;
+            const bool direct = in_i32(u0 * kap + lam) && in_i32(u1 * kap + lam);
+            long long ulo = 0, uhi = 0;
+            const bool clamp = !direct && saturation_bounds(kap, lam, sh, top, &ulo, &uhi);
+            const int mode = direct ? kModeDirect : clamp ? kModeClamp : kModeWide;
+            const uint32_t lam2 = beta * static_cast<uint32_t>(kap) + static_cast<uint32_t>(lam);
+            r0 = make_int4(static_cast<int32_t>(lam2), kap, sh, mode);
+            r1 = make_int4(static_cast<int32_t>(beta), static_cast<int32_t>(ulo), static_cast<int32_t>(uhi), lam);
+        }
+        rec0[o] = r0;
+        rec1[o] = r1;
+    }
+    epi_sync();
+    // one "all direct" flag per 16-channel group
+    uint8_t *gd = reinterpret_cast<uint8_t *>(rec1 + NT);
+    if (et < NT / 16) {
+        int all = 1;
+        for (int k = 0; k < 16; ++k) all &= rec0[et * 16 + k].w == kModeDirect;
+        gd[et] = static_cast<uint8_t>(all);
+    }
+    epi_sync();
+}
+
+// The prepared image: the loader's two bulk copies (B, then the tail) on w_full.
+__device__ __forceinline__ void load_image(const WinArgs &a, uint8_t *smem, uint64_t *w_full)
+{
+    if ((threadIdx.x & 31) == 0) {
+        mbar_arrive_expect_tx(w_full, a.b_bytes + a.tail_bytes);
+        for (uint32_t off = 0; off < a.b_bytes; off += 32768u)
+            bulk_g2s(smem + a.off_b + off, a.img + off, min(32768u, a.b_bytes - off), w_full);
+        for (uint32_t off = 0; off < a.tail_bytes; off += 32768u)
+            bulk_g2s(smem + a.off_rec + off, a.img + a.b_bytes + off, min(32768u, a.tail_bytes - off), w_full);
+    }
+    __syncwarp();
+}
+
+// Warps 4-12 with a prepared image: once it has landed, the slot layout
+// follows from the accumulator count it carries.
+template <int NT>
+__device__ __forceinline__ void image_ready(const WinArgs &a, uint8_t *smem, Misc *misc, uint64_t *w_full)
+{
+    mbar_wait_warp(w_full, 0, a.status);
+    if (threadIdx.x == kPrepWarp0 * 32) {
+        const int *spare = reinterpret_cast<const int *>(smem + a.off_tap) + (a.taps + 2) * NT;
+        const uint32_t nacc = static_cast<uint32_t>(spare[0]), cols = static_cast<uint32_t>(a.s) * nacc * NT;
+        misc->nch = nacc;
+        misc->kx = static_cast<uint32_t>(spare[1]);
+        misc->slot_cols = cols;
+        misc->nslots = min(static_cast<uint32_t>(kMaxSlots), 512u / cols);
+        misc->nmma = static_cast<uint32_t>(a.s * a.taps * a.ksteps);
+    }
+    prep_sync();
+}
+
+// Warps 4-12 after the preparation: B and the tail out to the image (16-byte units).
+__device__ __forceinline__ void store_image(const WinArgs &a, const uint8_t *smem)
+{
+    const int et = threadIdx.x - kPrepWarp0 * 32;
+    for (uint32_t off = static_cast<uint32_t>(et) * 16u; off < a.b_bytes; off += kPrepThreads * 16u)
+        *reinterpret_cast<uint4 *>(a.img_out + off) = *reinterpret_cast<const uint4 *>(smem + a.off_b + off);
+    for (uint32_t off = static_cast<uint32_t>(et) * 16u; off < a.tail_bytes; off += kPrepThreads * 16u)
+        *reinterpret_cast<uint4 *>(a.img_out + a.b_bytes + off) =
+            *reinterpret_cast<const uint4 *>(smem + a.off_rec + off);
 }
 
 // ---------------------------------------------------------------- epilogue (warps 4-11)
@@ -663,8 +750,10 @@ __device__ __forceinline__ void tmem_load(uint32_t addr, uint32_t (&v)[EB])
     if constexpr (EB >= 16) {
 #pragma unroll
         for (int b0 = 0; b0 < EB; b0 += 16) tmem_ld16(addr + b0, *reinterpret_cast<uint32_t(*)[16]>(v + b0));
-    } else {
+    } else if constexpr (EB == 8) {
         tmem_ld8(addr, *reinterpret_cast<uint32_t(*)[8]>(v));
+    } else {
+        tmem_ld4(addr, *reinterpret_cast<uint32_t(*)[4]>(v));
     }
 }
 
@@ -787,12 +876,11 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
         my_sh[r] = static_cast<uint32_t>(rec.z);
         direct_all = __all_sync(0xffffffffu, l_direct(gdirect, m)) && direct_all;
     }
+    // one shift for all of this warp's channels: the common case, one shuffle less per value
+    const uint32_t shift = __shfl_sync(0xffffffffu, my_sh[0], 0);
+    const bool one_shift = __all_sync(0xffffffffu, my_sh[0] == shift && my_sh[1] == shift);
     const uint32_t strip1 = static_cast<uint32_t>(nch) * NT;  // columns from strip 0's buffers to strip 1's
     int *const status = a.status;
-
-    // all slots start free (the MMA warp writes each accumulator's pre-load)
-    if (lane == 0)
-        for (int slot = 0; slot < nslots; ++slot) mbar_arrive(&acc_empty[slot]);
 
     const int oyr = row >> 3, oxr = row & 7;
     for (int i = 0, t = blockIdx.x; t < a.total_tiles; ++i, t += gridDim.x) {
@@ -838,13 +926,23 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
                 const int set = k0 >= 32 ? 1 : 0;
                 const uint32_t l2 = set ? my_lam2[1] : my_lam2[0], kp = set ? my_kap[1] : my_kap[0];
                 const uint32_t shv = set ? my_sh[1] : my_sh[0];
+                if (one_shift) {
 #pragma unroll
-                for (int k = 0; k < EB; ++k) {
-                    const uint32_t lam2 = __shfl_sync(0xffffffffu, l2, (k0 + k) & 31);
-                    const uint32_t kap = __shfl_sync(0xffffffffu, kp, (k0 + k) & 31);
-                    const uint32_t sh = __shfl_sync(0xffffffffu, shv, (k0 + k) & 31);
-                    y0[k] = static_cast<int32_t>(v0[k] * kap + lam2) >> sh;
-                    y1[k] = static_cast<int32_t>(v1[k] * kap + lam2) >> sh;
+                    for (int k = 0; k < EB; ++k) {
+                        const uint32_t lam2 = __shfl_sync(0xffffffffu, l2, (k0 + k) & 31);
+                        const uint32_t kap = __shfl_sync(0xffffffffu, kp, (k0 + k) & 31);
+                        y0[k] = static_cast<int32_t>(v0[k] * kap + lam2) >> shift;
+                        y1[k] = static_cast<int32_t>(v1[k] * kap + lam2) >> shift;
+                    }
+                } else {
+#pragma unroll
+                    for (int k = 0; k < EB; ++k) {
+                        const uint32_t lam2 = __shfl_sync(0xffffffffu, l2, (k0 + k) & 31);
+                        const uint32_t kap = __shfl_sync(0xffffffffu, kp, (k0 + k) & 31);
+                        const uint32_t sh = __shfl_sync(0xffffffffu, shv, (k0 + k) & 31);
+                        y0[k] = static_cast<int32_t>(v0[k] * kap + lam2) >> sh;
+                        y1[k] = static_cast<int32_t>(v1[k] * kap + lam2) >> sh;
+                    }
                 }
             } else {
 #pragma unroll
@@ -902,24 +1000,44 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     __syncthreads();
     tc_fence_after();
 
-    // The loader starts the copies (filters, then the first windows); the whole
-    // block prepares the filters; then each warp takes its role.
-    LoadState ld{0, 0, static_cast<int>(blockIdx.x), 0u};
-    if (warp == kLoadWarp) {
-        load_filters(a, smem, w_full);
-        load_windows(a, smem, raw_full, raw_empty, ld, a.raw_stages);
-    }
-    prepare_filters<BITS, NT>(a, smem, misc, w_full);
-
+    // Each warp takes its role.  The loader copies the filters (or the
+    // prepared image), then streams the windows; the converters stage windows
+    // from the start; the epilogue warps and the MMA warp first prepare the
+    // filters together (or wait for the image).  With img_out the block only
+    // prepares the filters and writes the image.
+    const bool convolve = a.img_out == nullptr;
     if (warp < kConvWarps) {
-        converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
-    } else if (warp < kConvWarps + kEpiWarps) {
-        epilogue_role<BITS, NT, POOL>(a, smem, acc_full, acc_empty, misc);
-    } else if (warp == kMmaWarp) {
-        mma_role<NT, BITS != 8>(a, smem, a_full, a_empty, acc_full, acc_empty, done, misc);
+        if (convolve) converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
     } else if (warp == kLoadWarp) {
-        load_windows(a, smem, raw_full, raw_empty, ld, a.total_tiles);
-        load_drain(a, raw_full, w_full, ld);
+        if (a.img) {
+            load_image(a, smem, w_full);
+        } else {
+            load_filters(a, smem, w_full);
+        }
+        if (convolve) {
+            LoadState ld{0, 0, static_cast<int>(blockIdx.x), 0u};
+            load_windows(a, smem, raw_full, raw_empty, ld, a.total_tiles);
+            load_drain(a, raw_full, w_full, ld);
+        }
+    } else {
+        if (a.img) {
+            image_ready<NT>(a, smem, misc, w_full);
+        } else {
+            prepare_filters<BITS, NT>(a, smem, misc, w_full);
+        }
+        if (warp == kMmaWarp) {
+            if (convolve) mma_role<NT, BITS != 8>(a, smem, a_full, a_empty, acc_full, acc_empty, done, misc);
+        } else {
+            // all slots start free (the MMA warp writes each accumulator's pre-load)
+            if (convolve && (threadIdx.x & 31) == 0)
+                for (uint32_t slot = 0; slot < misc->nslots; ++slot) mbar_arrive(&acc_empty[slot]);
+            if (!a.img) prepare_records<BITS, NT>(a, smem, misc);
+            if (convolve) epilogue_role<BITS, NT, POOL>(a, smem, acc_full, acc_empty, misc);
+        }
+        if (!convolve) {
+            prep_sync();
+            store_image(a, smem);
+        }
     }
 
     tc_fence_before();

@@ -98,21 +98,21 @@ struct WinPlan {
     uint32_t raw_row_bytes, raw_bytes, b_bytes, chunk_stride, stage_bytes;
     uint32_t off_b, off_a, off_raw, off_rec, off_thr, off_tap, off_mtab, off_pre, off_wraw, off_bar, smem_bytes;
     uint32_t wraw_bytes;  // packed filters bulk-copied into shared memory (0: read from global memory)
-    size_t param_bytes;   // qconv_hwc_prepare workspace: copies of the filters and constants
-    size_t off_pw, off_pbias, off_pkappa, off_plambda, off_pshifts, off_pthr;  // within it
+    uint32_t tail_bytes;  // shared memory from off_rec to the end of the pre-load operands
+    size_t img_bytes;     // qconv_hwc_prepare workspace: the prepared image (B, then the tail)
 };
 
 WinPlan plan_conv_win(const ConvShape &s);
-// One launch: the window kernel reads the caller's filters and constants (p.w,
-// p.bias, ...), or copies of them that qconv_hwc_prepare placed in a workspace.
-cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, cudaStream_t st);
-// qconv_hwc_prepare for the window kernel: copies filters and constants into
-// the workspace (device-to-device copies on `st`), laid out as the plan says.
+// One launch of the window kernel.  With img == nullptr it prepares the
+// caller's filters and constants (p.w, p.bias, ...) itself; with img it reads
+// the image qconv_hwc_prepare wrote (img_bytes at img) and p carries only x, y.
+cudaError_t launch_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, cudaStream_t st,
+                            const void *img = nullptr);
+// qconv_hwc_prepare for the window kernel: one block prepares the filters and
+// constants exactly as a convolving launch would and writes the image
+// (plan.img_bytes) to `workspace`.
 cudaError_t prepare_conv_win(const WinPlan &plan, const ConvShape &s, const ConvParams &p, void *workspace,
                              cudaStream_t st);
-// ConvParams pointing at the copies in a prepared workspace (bias and per-channel
-// shifts always present there: zeros and the scalar shift when the caller gave none).
-ConvParams win_prepared_params(const WinPlan &plan, const void *workspace);
 
 // ---- max-pool, fully connected, packing
 cudaError_t launch_maxpool(int n, int h, int w, int c, int k, int s, int bits, const uint8_t *x, uint8_t *y,

@@ -152,8 +152,10 @@ def test_subbyte_layers_with_c_multiple_of_32_plan_e4m3_filters(lib):
 def test_window_kernel_selection_and_prepared_workspace(lib):
     """Tensor-core requests take the window kernel where its plan fits (the benchmark layer at
     every Q, the CIFAR-shaped conv2 / conv3) and the general kernel elsewhere (C = 3, more than
-    128 output channels).  The window kernel's prepared workspace holds copies of the packed
-    filters, bias, kappa, lambda and shifts, each 256-byte aligned."""
+    128 output channels).  The window kernel's prepared workspace holds the image qconv_hwc_prepare
+    builds: the filters as the B operand (taps x 4 K-chunks x 64 rows x 16 bytes), then the
+    records (2 x 64 x 16 bytes + flags), the tap sums ((taps + 3) x 64 int32), the MMA table
+    (2 strips x 9 taps x 2 k-steps x 8 bytes) and the pre-load operands (4 KB + 64 x 32 bytes)."""
     for bits in (8, 4, 2):
         assert qnn.tc_kernel(desc(bits=bits)) == qnn.ALGO_TC_WINDOW
     assert qnn.tc_kernel(qnn.conv_desc(1024, 16, 16, 32, 32, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_WINDOW
@@ -162,10 +164,9 @@ def test_window_kernel_selection_and_prepared_workspace(lib):
     assert qnn.tc_kernel(qnn.conv_desc(64, 14, 14, 256, 512, 1, 1, 1, 0, 8, 10)) == qnn.ALGO_TC_GENERAL
     assert qnn.tc_kernel(desc(algo=qnn.ALGO_TC_GENERAL)) == qnn.ALGO_TC_GENERAL
     assert qnn.tc_kernel(desc(stride=(2, 2))) == 0
-    # 64 x 3x3x32 bytes of filters, then int32 bias, int16 kappa, int32 lambda, uint8 shifts
-    r = lambda v: (v + 255) // 256 * 256  # noqa: E731
-    wbytes = 64 * 9 * 32
-    assert qnn.workspace_size(desc()) == r(r(r(r(wbytes) + 4 * 64) + 2 * 64) + 4 * 64) + 256
+    parts = 9 * 4 * 64 * 16 + (2 * 64 * 16 + 16) + 12 * 64 * 4 + 2 * 9 * 2 * 8 + 4096 + 64 * 32
+    size = qnn.workspace_size(desc())
+    assert size % 256 == 0 and parts <= size <= parts + 256 + 128  # 16- and 128-byte region alignment
 
 
 def test_other_entry_points_validate(lib):

@@ -91,6 +91,9 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
         const int ct = (p.taps + nch - 1) / nch, last_len = p.taps - (nch - 1) * ct;
         if (last_len <= 0) continue;  // the kernel never takes a split with an empty chunk
         const int nmma = p.s * p.taps * p.ksteps;
+        // K-split (the kernel's rule): k-step kk of a tap goes to accumulator kk % kx of its chunk
+        const int kx = (p.s * nch == 1 && p.ksteps % 2 == 0 && 2 * p.nt <= 256) ? 2 : 1;
+        CHECK(p.s * nch * kx * p.nt <= 512, "slot with the K-split");
         std::vector<int> seen(nmma, 0), unit(p.taps * p.ksteps * p.s, 0);
         CHECK(ct * p.ksteps <= 256, "one step pair per preparation thread");
         for (int et = 0; et < ct * p.ksteps; ++et) {
@@ -105,7 +108,7 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
                     CHECK(u >= 0 && u < nmma, "table index %d", u);
                     if (u >= 0 && u < nmma) ++seen[u];
                     ++unit[(tap * p.ksteps + kk) * p.s + sj];
-                    CHECK((sj * nch + cc) * p.nt + p.nt <= 512, "accumulator column");
+                    CHECK(((sj * nch + cc) * kx + kk % kx) * p.nt + p.nt <= p.s * nch * kx * p.nt, "accumulator column");
                     CHECK(8LL * nmma <= 8LL * p.s * p.taps * p.ksteps, "table size");
                 }
             }
