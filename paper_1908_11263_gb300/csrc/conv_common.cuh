@@ -242,8 +242,13 @@ __device__ __forceinline__ void store_packed(const uint32_t (&packed)[(G * BITS 
 {
     constexpr int kWords = (G * BITS + 31) / 32;
     constexpr int kBytes = G * BITS / 8;
-    if (valid >= G && (reinterpret_cast<uintptr_t>(dst) % kBytes) == 0) {
-        if (kBytes == 16) *reinterpret_cast<uint4 *>(dst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    if (valid >= G && (reinterpret_cast<uintptr_t>(dst) % (kBytes < 16 ? kBytes : 16)) == 0) {
+        if (kBytes >= 16) {
+#pragma unroll
+            for (int q = 0; q < kBytes / 16; ++q)
+                reinterpret_cast<uint4 *>(dst)[q] =
+                    make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+        }
         else if (kBytes == 8) *reinterpret_cast<uint2 *>(dst) = make_uint2(packed[0], packed[kWords > 1 ? 1 : 0]);
         else if (kBytes == 4) *reinterpret_cast<uint32_t *>(dst) = packed[0];
         else if (kBytes == 2) *reinterpret_cast<uint16_t *>(dst) = static_cast<uint16_t>(packed[0]);

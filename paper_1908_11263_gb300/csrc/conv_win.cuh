@@ -81,8 +81,24 @@ struct Misc {
     uint32_t mask;
     uint32_t nmma;  // MMAs per tile (entries of the issue table)
     uint32_t kx;    // K-split: the k-steps of a tap alternate between kx accumulators
-    uint32_t pad;
+    uint32_t cst;   // TMEM column of the per-channel constants (lam2, then kappa), or ~0u: none
 };
+
+// Accumulator slots of `cols` columns each, and the 2 * NT columns of the
+// per-channel constants behind them when two slots still fit.
+template <int NT>
+__device__ __forceinline__ void slot_layout(Misc *misc, uint32_t cols)
+{
+    uint32_t ns = min(static_cast<uint32_t>(kMaxSlots), (512u - 2u * NT) / cols);
+    uint32_t cst = ns * cols;
+    if (ns < 2) {
+        ns = min(static_cast<uint32_t>(kMaxSlots), 512u / cols);
+        cst = ~0u;
+    }
+    misc->slot_cols = cols;
+    misc->nslots = ns;
+    misc->cst = cst;
+}
 
 struct WinArgs {
     const uint8_t *x;
@@ -624,8 +640,7 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
         // the tap area's spare row carries both into a prepared image
         tapabs[(a.taps + 2) * NT] = nch * kx;
         tapabs[(a.taps + 2) * NT + 1] = kx;
-        misc->slot_cols = cols;
-        misc->nslots = min(static_cast<uint32_t>(kMaxSlots), 512u / cols);
+        slot_layout<NT>(misc, cols);
         misc->nmma = static_cast<uint32_t>(a.s * a.taps * a.ksteps);
     }
     // B and the pre-load operands were written through the generic proxy; the
@@ -720,8 +735,7 @@ __device__ __forceinline__ void image_ready(const WinArgs &a, uint8_t *smem, Mis
         const uint32_t nacc = static_cast<uint32_t>(spare[0]), cols = static_cast<uint32_t>(a.s) * nacc * NT;
         misc->nch = nacc;
         misc->kx = static_cast<uint32_t>(spare[1]);
-        misc->slot_cols = cols;
-        misc->nslots = min(static_cast<uint32_t>(kMaxSlots), 512u / cols);
+        slot_layout<NT>(misc, cols);
         misc->nmma = static_cast<uint32_t>(a.s * a.taps * a.ksteps);
     }
     prep_sync();
@@ -839,15 +853,136 @@ __device__ __forceinline__ void store_block(const int (&y)[EB], bool store, int 
     if (store) store_packed<BITS, EB>(pk, valid, dst);
 }
 
+// HB packed Q-bit values of one strip's pixel (whole words when HB * Q is a
+// multiple of 32, else the low bits of one word): max-pooled over the 2x2
+// window when POOL (every lane shuffles), stored.
+template <int BITS, int HB, bool POOL>
+__device__ __forceinline__ void store_words(uint32_t (&pk)[(HB * BITS + 31) / 32 < 1 ? 1 : (HB * BITS + 31) / 32],
+                                            bool store, int valid, uint8_t *dst)
+{
+    if constexpr (POOL) {
+#pragma unroll
+        for (int wd = 0; wd < (HB * BITS + 31) / 32; ++wd) {
+            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 1));
+            pk[wd] = max_fields<BITS>(pk[wd], __shfl_xor_sync(0xffffffffu, pk[wd], 8));
+        }
+    }
+    if (store) store_packed<BITS, HB>(pk, valid, dst);
+}
+
 // Whether channel m's compression is in the direct form (flags per 16 channels).
 __device__ __forceinline__ bool l_direct(const uint8_t *gdirect, int m) { return gdirect[m >> 4] != 0; }
+
+// One tile's epilogue state for a warp: its TMEM columns, channels, output
+// pixels and whether the direct form with one shift covers all its channels.
+template <int NT>
+struct EpiTile {
+    uint32_t base, strip1;
+    bool two;
+    int nch, col0, lane;
+    bool direct_all, one_shift;
+    uint32_t shift;
+    const int4 *rec0, *rec1;
+    uint8_t *dst[2];
+    bool store[2];
+    uint64_t *acc_empty;
+    bool tmem_cst;     // lam2 and kappa of the block's channels come from TMEM with the accumulators
+    uint32_t cst_addr; // TMEM address of lam2 of channel col0 in this warp's lanes (kappa NT columns on)
+};
+
+// The tile's columns in blocks of HB: the loads of a block (NCH accumulators
+// per strip, 0 = any count, one wait per accumulator), the slot released
+// after the last block's loads, then compression, packing and stores (HB
+// values of a pixel are HB * Q / 8 contiguous bytes).
+template <int BITS, int NT, bool POOL, int HB, int NCH>
+__device__ __forceinline__ void epi_tile(const WinArgs &a, const EpiTile<NT> &e, const uint32_t (&my_lam2)[2],
+                                         const uint32_t (&my_kap)[2], const uint32_t (&my_sh)[2])
+{
+    constexpr int CW = NT / 2;
+#pragma unroll 1
+    for (int k0 = 0; k0 < CW; k0 += HB) {
+        uint32_t v0[HB], v1[HB], cl[HB], ck[HB];  // accumulators; lam2 and kappa when tmem_cst
+        if constexpr (NCH == 0) {
+            drain_many<HB>(e.base + k0, e.base + e.strip1 + k0, e.two, e.nch, NT, v0, v1);
+        } else {
+            uint32_t t0[NCH == 2 ? HB : 1], t1[NCH == 2 ? HB : 1];
+            if (e.tmem_cst) {
+                tmem_load<HB>(e.cst_addr + k0, cl);
+                tmem_load<HB>(e.cst_addr + NT + k0, ck);
+            }
+            tmem_load<HB>(e.base + k0, v0);
+            if constexpr (NCH == 2) tmem_load<HB>(e.base + k0 + NT, t0);
+            if (e.two) {
+                tmem_load<HB>(e.base + e.strip1 + k0, v1);
+                if constexpr (NCH == 2) tmem_load<HB>(e.base + e.strip1 + k0 + NT, t1);
+            }
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < HB; ++k) {
+                asm volatile("" : "+r"(v0[k]), "+r"(v1[k]), "+r"(cl[k]), "+r"(ck[k]));  // uses stay after the wait
+                if constexpr (NCH == 2) {
+                    asm volatile("" : "+r"(t0[k]), "+r"(t1[k]));
+                    v0[k] += t0[k];
+                    v1[k] += t1[k];  // unused when !two
+                }
+            }
+        }
+        if (k0 + HB >= CW) {  // the slot's last columns are read: give it back first
+            tc_fence_before();
+            __syncwarp();
+            if (e.lane == 0) mbar_arrive(e.acc_empty);
+        }
+        const int m0 = e.col0 + k0;
+        const int valid = a.m - m0;  // same for the whole warp
+        if (valid <= 0) continue;
+        // groups of 8 channels: their constants, both strips' values, packed at once
+        constexpr int kG = HB < (BITS == 2 ? 16 : 8) ? HB : (BITS == 2 ? 16 : 8);  // a whole number of words
+        constexpr int kGW = (kG * BITS + 31) / 32;  // packed words per group
+        uint32_t pk0[HB / kG * kGW], pk1[HB / kG * kGW];
+#pragma unroll
+        for (int g0 = 0; g0 < HB; g0 += kG) {
+            int y0[kG], y1[kG];
+            if (NCH != 0 && e.tmem_cst) {
+                // direct form, one shift: the constants arrived with the accumulators
+#pragma unroll
+                for (int k = 0; k < kG; ++k) {
+                    y0[k] = static_cast<int32_t>(v0[g0 + k] * ck[g0 + k] + cl[g0 + k]) >> e.shift;
+                    y1[k] = static_cast<int32_t>(v1[g0 + k] * ck[g0 + k] + cl[g0 + k]) >> e.shift;
+                }
+            } else if (e.direct_all) {
+                // direct channels: ((s * kappa + lam2) mod 2^32) >> shift is exact (see the records);
+                // the constants of channel col0 + k0 + k sit in lane (k0 + k) % 32 of set (k0 + k) / 32
+#pragma unroll
+                for (int k = 0; k < kG; ++k) {
+                    const int c = k0 + g0 + k, set = c >= 32 ? 1 : 0;
+                    const uint32_t lam2 = __shfl_sync(0xffffffffu, set ? my_lam2[1] : my_lam2[0], c & 31);
+                    const uint32_t kap = __shfl_sync(0xffffffffu, set ? my_kap[1] : my_kap[0], c & 31);
+                    const uint32_t sh =
+                        e.one_shift ? e.shift : __shfl_sync(0xffffffffu, set ? my_sh[1] : my_sh[0], c & 31);
+                    y0[k] = static_cast<int32_t>(v0[g0 + k] * kap + lam2) >> sh;
+                    y1[k] = static_cast<int32_t>(v1[g0 + k] * kap + lam2) >> sh;
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < kG; ++k) {
+                    const int4 r0 = e.rec0[m0 + g0 + k], r1 = e.rec1[m0 + g0 + k];
+                    y0[k] = static_cast<int>(compress_slow(v0[g0 + k], r0, r1, (1u << BITS) - 1u));
+                    y1[k] = e.two ? static_cast<int>(compress_slow(v1[g0 + k], r0, r1, (1u << BITS) - 1u)) : 0;
+                }
+            }
+            pack_values<BITS, kG>(y0, *reinterpret_cast<uint32_t(*)[kGW]>(pk0 + g0 / kG * kGW));
+            pack_values<BITS, kG>(y1, *reinterpret_cast<uint32_t(*)[kGW]>(pk1 + g0 / kG * kGW));
+        }
+        store_words<BITS, HB, POOL>(pk0, e.store[0], valid, e.dst[0] + m0 * BITS / 8);
+        if (e.two) store_words<BITS, HB, POOL>(pk1, e.store[1], valid, e.dst[1] + m0 * BITS / 8);
+    }
+}
 
 template <int BITS, int NT, bool POOL>
 __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, uint64_t *acc_full, uint64_t *acc_empty,
                                               const Misc *misc)
 {
     constexpr int CW = NT / 2;             // columns of this warp
-    constexpr int EB = CW < 8 ? CW : 8;    // columns drained and compressed together (2 strips x 2 chunks in flight)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quarter = warp & 3, half = (warp - kEpiWarp0) >> 2;
     const int row = quarter * 32 + lane;  // tile row of a strip: 8 * (output row) + column
@@ -881,6 +1016,28 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
     const bool one_shift = __all_sync(0xffffffffu, my_sh[0] == shift && my_sh[1] == shift);
     const uint32_t strip1 = static_cast<uint32_t>(nch) * NT;  // columns from strip 0's buffers to strip 1's
     int *const status = a.status;
+    // The direct-form constants of this warp's channels, one row per lane of its
+    // quarter (all rows alike): the block loop reads them with the accumulators
+    // instead of broadcasting them lane to lane (shuffles queue behind the
+    // tensor cores' shared-memory reads).
+    const uint32_t cst = misc->cst;
+    const bool tmem_cst = cst != ~0u && direct_all && one_shift;
+    const uint32_t cst_addr = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + cst + col0;
+    if (tmem_cst) {
+#pragma unroll 1
+        for (int j = 0; j < CW; j += 16) {
+            uint32_t l[16], kp[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                const int4 r = rec0[col0 + j + k];
+                l[k] = static_cast<uint32_t>(r.x);
+                kp[k] = static_cast<uint32_t>(r.y);
+            }
+            tmem_st16(cst_addr + j, l);
+            tmem_st16(cst_addr + NT + j, kp);
+        }
+        tmem_wait_st();
+    }
 
     const int oyr = row >> 3, oxr = row & 7;
     for (int i = 0, t = blockIdx.x; t < a.total_tiles; ++i, t += gridDim.x) {
@@ -907,54 +1064,15 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
             store[s] = store[s] && (s == 0 || two);
         }
         const uint32_t base = lane_addr + slot * slot_cols;
-#pragma unroll 1
-        for (int k0 = 0; k0 < CW; k0 += EB) {
-            uint32_t v0[EB], v1[EB];
-            drain_block<EB>(base + k0, base + strip1 + k0, two, nch, NT, v0, v1);
-            if (k0 + EB == CW) {  // the slot's last columns are read: give it back first
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&acc_empty[slot]);
-            }
-            const int m0 = col0 + k0;
-            const int valid = a.m - m0;  // same for the whole warp
-            if (valid <= 0) continue;
-            int y0[EB], y1[EB];
-            if (direct_all) {
-                // direct channels: ((s * kappa + lam2) mod 2^32) >> shift is exact (see the records);
-                // the constants of channel col0 + k0 + k sit in lane (k0 + k) % 32 of set (k0 + k) / 32
-                const int set = k0 >= 32 ? 1 : 0;
-                const uint32_t l2 = set ? my_lam2[1] : my_lam2[0], kp = set ? my_kap[1] : my_kap[0];
-                const uint32_t shv = set ? my_sh[1] : my_sh[0];
-                if (one_shift) {
-#pragma unroll
-                    for (int k = 0; k < EB; ++k) {
-                        const uint32_t lam2 = __shfl_sync(0xffffffffu, l2, (k0 + k) & 31);
-                        const uint32_t kap = __shfl_sync(0xffffffffu, kp, (k0 + k) & 31);
-                        y0[k] = static_cast<int32_t>(v0[k] * kap + lam2) >> shift;
-                        y1[k] = static_cast<int32_t>(v1[k] * kap + lam2) >> shift;
-                    }
-                } else {
-#pragma unroll
-                    for (int k = 0; k < EB; ++k) {
-                        const uint32_t lam2 = __shfl_sync(0xffffffffu, l2, (k0 + k) & 31);
-                        const uint32_t kap = __shfl_sync(0xffffffffu, kp, (k0 + k) & 31);
-                        const uint32_t sh = __shfl_sync(0xffffffffu, shv, (k0 + k) & 31);
-                        y0[k] = static_cast<int32_t>(v0[k] * kap + lam2) >> sh;
-                        y1[k] = static_cast<int32_t>(v1[k] * kap + lam2) >> sh;
-                    }
-                }
-            } else {
-#pragma unroll
-                for (int k = 0; k < EB; ++k) {
-                    const int4 r0 = rec0[m0 + k], r1 = rec1[m0 + k];
-                    y0[k] = static_cast<int>(compress_slow(v0[k], r0, r1, (1u << BITS) - 1u));
-                    y1[k] = two ? static_cast<int>(compress_slow(v1[k], r0, r1, (1u << BITS) - 1u)) : 0;
-                }
-            }
-            store_block<BITS, EB, POOL>(y0, store[0], valid, dst[0] + m0 * BITS / 8);
-            if (two) store_block<BITS, EB, POOL>(y1, store[1], valid, dst[1] + m0 * BITS / 8);
-        }
+        const EpiTile<NT> et{base,     strip1,  two,   nch,  col0,     lane,
+                             direct_all, one_shift, shift, rec0, rec1,  {dst[0], dst[1]},
+                             {store[0], store[1]}, &acc_empty[slot], tmem_cst, cst_addr};
+        // every load of a block of 8 columns (both strips' accumulators and, with
+        // tmem_cst, the constants) goes out before one wait; more than two
+        // accumulators per strip: one wait per accumulator
+        if (nch == 1) epi_tile<BITS, NT, POOL, (CW < 8 ? CW : 8), 1>(a, et, my_lam2, my_kap, my_sh);
+        else if (nch == 2) epi_tile<BITS, NT, POOL, (CW < 8 ? CW : 8), 2>(a, et, my_lam2, my_kap, my_sh);
+        else epi_tile<BITS, NT, POOL, (CW < 8 ? CW : 8), 0>(a, et, my_lam2, my_kap, my_sh);
     }
 }
 
