@@ -1093,6 +1093,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     uint64_t *w_full = done + 1;
     Misc *misc = reinterpret_cast<Misc *>(w_full + 2);  // (one spare barrier slot)
     const int warp = threadIdx.x >> 5;
+    // Programmatic dependent launch: the next kernel in the stream may launch
+    // now; its blocks take each SM as this kernel's block there exits, and do
+    // their setup while the rest of this grid finishes.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp == kMmaWarp) {
         if ((threadIdx.x & 31) == 0) {
@@ -1117,6 +1121,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // nothing above reads global memory: from here on, everything the previous
+    // kernel in the stream wrote is visible
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     // Each warp takes its role.  The loader copies the filters (or the
     // prepared image), then streams the windows; the converters stage windows

@@ -32,8 +32,19 @@ cudaError_t launch_one(const win::WinArgs &a, int grid, uint32_t smem, cudaStrea
             raised[dev] = true;
         }
     }
-    kern<<<grid, win::kThreads, smem, st>>>(a);
-    return cudaGetLastError();
+    // launched with programmatic stream serialization: the kernel lets its
+    // successor launch early and waits for its predecessor before reading memory
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(win::kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 }  // namespace
