@@ -141,7 +141,12 @@ qnn_status qconv_hwc(const qnn_conv_desc *d, const void *x, const void *w, const
  * qconv_hwc_run: the convolution itself, reading a workspace prepared for the
  *   same descriptor (any other workspace content gives undefined results).
  *   Only for descriptors that select the tensor-core kernel; otherwise
- *   QNN_EUNSUPPORTED.
+ *   QNN_EUNSUPPORTED.  The window kernel launches with programmatic stream
+ *   serialization: it may start while the previous kernel in the stream is
+ *   still running, waits for it before touching x or y, and reads the
+ *   workspace before that wait, so the workspace must not be written by the
+ *   kernel launched just before it (qconv_hwc_prepare's own launch is fine:
+ *   its successor starts only after it ends).
  * qconv_hwc(...) is exactly qconv_hwc_prepare(...) followed by qconv_hwc_run(...)
  * on the same stream.
  */

@@ -1095,8 +1095,11 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     const int warp = threadIdx.x >> 5;
     // Programmatic dependent launch: the next kernel in the stream may launch
     // now; its blocks take each SM as this kernel's block there exits, and do
-    // their setup while the rest of this grid finishes.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // their setup while the rest of this grid finishes.  A launch that writes
+    // a prepared image (img_out) does not: its successor starts after it ends,
+    // so a convolving launch may read its image before waiting on its
+    // predecessor (every image was written by an earlier, finished launch).
+    if (a.img_out == nullptr) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp == kMmaWarp) {
         if ((threadIdx.x & 31) == 0) {
@@ -1121,8 +1124,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    // nothing above reads global memory: from here on, everything the previous
-    // kernel in the stream wrote is visible
+    // the prepared image comes from a finished launch: its copy may start now
+    if (warp == kLoadWarp && a.img) load_image(a, smem, w_full);
+    // nothing above reads other global memory: from here on, everything the
+    // previous kernel in the stream wrote is visible
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
     // Each warp takes its role.  The loader copies the filters (or the
@@ -1134,11 +1139,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     if (warp < kConvWarps) {
         if (convolve) converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
     } else if (warp == kLoadWarp) {
-        if (a.img) {
-            load_image(a, smem, w_full);
-        } else {
-            load_filters(a, smem, w_full);
-        }
+        if (!a.img) load_filters(a, smem, w_full);
         if (convolve) {
             LoadState ld{0, 0, static_cast<int>(blockIdx.x), 0u};
             load_windows(a, smem, raw_full, raw_empty, ld, a.total_tiles);
