@@ -5,9 +5,9 @@ import numpy as np
 import pytest
 import torch
 
-from paper_1908_11263_gb300 import qnn
+from paper_1908_11263_gb300 import inputs, qnn
 
-from gpu_util import conv_gpu, conv_oracle, first_mismatch, pack_gpu, tc_algos, to_dev
+from gpu_util import conv_gpu, conv_oracle, dev, first_mismatch, layer_tensors, pack_gpu, tc_algos, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -112,3 +112,53 @@ def test_prepared_path(algo, bits, with_bias_and_shifts):
         qnn.device_status()
         assert first_mismatch(got, want) is None, (trial, first_mismatch(got, want))
         assert len(np.unique(want)) > 4
+
+
+@pytest.mark.parametrize("which", ["w2", "w4_int4", "w4_int2"])
+def test_prepared_graph_full_size(which):
+    """The launch configuration bench.py times, at the benchmark layer's full size (batch 512):
+    filters prepared once, then qconv_hwc_run launches captured back to back in a CUDA graph on a
+    side stream (consecutive launches overlap through programmatic dependent launch), alternating
+    between two inputs and four outputs.  Every output byte equals the oracle's."""
+    if which == "w2":
+        (key, layer, wl, lid), = inputs.single_layer_workload(inputs.WORKLOAD_BATCH)
+    else:
+        (key, layer, wl, lid), = [t for t in inputs.single_layer_workload(inputs.WORKLOAD_SUBBYTE) if t[0] == which]
+    ld = inputs.make_layer(key, layer, wl, lid)
+    x, wt, bias, kappa, lam, shifts, shift = layer_tensors(ld)
+    bits, n = layer.bits, layer.n
+    st, pd = (layer.stride, layer.stride), (layer.pad, layer.pad)
+    want = conv_oracle(x, wt, bias, kappa, lam, shifts, shift, bits, st, pd)
+    want = want.reshape(n, -1)
+    assert len(np.unique(want)) > 4
+    per = 8 // bits
+    xs = [pack_gpu(x, bits).view(n, layer.h, layer.w, layer.c // per)]
+    xs.append(torch.flip(xs[0], dims=[0]).contiguous())  # the batch reversed: outputs reverse with it
+    wd = pack_gpu(wt, bits).view(layer.m, layer.k, layer.k, layer.c // per)
+    if bits == 8:
+        wd = wd.view(torch.int8)
+    stream = torch.cuda.Stream()
+    prep = qnn.PreparedConv(wd, to_dev(kappa, torch.int16), to_dev(lam, torch.int32), n=n, h=layer.h, wd=layer.w,
+                            bias=None if bias is None else to_dev(bias, torch.int32),
+                            shifts=None if shifts is None else to_dev(shifts, torch.uint8), shift=shift, bits=bits,
+                            stride=layer.stride, pad=layer.pad, stream=stream)
+    assert qnn.tc_kernel(prep.desc) == qnn.ALGO_TC_WINDOW
+    ys = [torch.full(prep.out_shape, 0xA5, dtype=torch.uint8, device=dev()) for _ in range(4)]
+    with torch.cuda.stream(stream):
+        prep(xs[0], out=ys[0], stream=stream)  # eager warm-up launch
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(8):
+            prep(xs[i % 2], out=ys[i % 4], stream=stream)
+    for y in ys:
+        y.fill_(0xA5)
+    torch.cuda.synchronize()
+    g.replay()
+    g.replay()
+    torch.cuda.synchronize()
+    qnn.device_status()
+    for i, y in enumerate(ys):
+        got = y.cpu().numpy().reshape(n, -1)
+        exp = want if i % 2 == 0 else want[::-1]
+        assert first_mismatch(got.reshape(-1), np.ascontiguousarray(exp).reshape(-1)) is None, (which, i)
