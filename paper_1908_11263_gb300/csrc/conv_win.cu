@@ -32,14 +32,19 @@ WinPlan plan_conv_win(const ConvShape &s)
     if (s.sh != 1 || s.sw != 1 || s.oh <= 0 || s.ow <= 0 || s.n < 0) return p;
     p.fp8 = s.bits != 8;
     p.kch = p.fp8 ? 16 : 8;
+    // INT-8 with few channels (C * kw <= 16, C not a multiple of 8): a kernel row's kw * C
+    // values of a position fill one 16-value K-step (two K-chunks)
+    p.fold = s.bits == 8 && s.c % 8 != 0 && s.kw > 1 && s.c * s.kw <= 16;
+    p.kwf = p.fold ? 1 : s.kw;
     // INT-8 in fp16 (whole 8-channel chunks), INT-4 / INT-2 in e4m3 (whole 32-channel pairs)
-    if (s.bits == 8 ? (s.c % 8 != 0) : (s.c % 32 != 0)) return p;
+    if (!p.fold && (s.bits == 8 ? (s.c % 8 != 0) : (s.c % 32 != 0))) return p;
     if (s.m > 128) return p;  // one filter set, all output channels in one MMA N
     p.nt = s.m <= 32 ? 32 : s.m <= 64 ? 64 : 128;
-    p.c_pad = (s.c + 2 * p.kch - 1) / (2 * p.kch) * (2 * p.kch);
+    // staged values per position and "tap" (a tap is a kernel row when folded)
+    p.c_pad = p.fold ? 16 : (s.c + 2 * p.kch - 1) / (2 * p.kch) * (2 * p.kch);
     p.groups = p.c_pad / p.kch;
     if (p.groups > 8) return p;  // the window holds every channel of a pixel
-    p.taps = s.kh * s.kw;
+    p.taps = p.fold ? s.kh : s.kh * s.kw;
     if (s.kh > 8 || s.kw > 8 || p.taps > win::kMaxTaps) return p;
     p.ksteps = p.groups / 2;
     const long long cb = static_cast<long long>(s.c) * s.bits / 8;
@@ -56,10 +61,11 @@ WinPlan plan_conv_win(const ConvShape &s)
         // into one TMEM buffer issue back to back at the full rate)
         const int nmin = 1;
         if (S * std::max(nmin, p.nch_max) * p.nt > 512) continue;  // one slot of accumulators in TMEM
-        const int sp = win::kCols * S + s.kw - 1, wh = win::kRows + s.kh - 1;
+        // folded positions carry their kw - 1 right neighbours: no extra window columns
+        const int sp = win::kCols * S + (p.fold ? 0 : s.kw - 1), wh = win::kRows + s.kh - 1;
         if (wh * sp > win::kMaxKP * 128) continue;  // converter positions per thread
         const int tiles_x = (s.ow + win::kCols * S - 1) / (win::kCols * S);
-        const bool full_rows = tiles_x == 1;
+        const bool full_rows = tiles_x == 1 || p.fold;  // folded windows read whole rows
         const long long row_bytes = s.w * cb;
         uint32_t raw_row_bytes;
         if (full_rows) {
@@ -82,7 +88,7 @@ WinPlan plan_conv_win(const ConvShape &s)
         const uint32_t mtab_bytes = round_up(static_cast<uint32_t>(S * p.taps * p.ksteps * 8), 16);
         const uint32_t pre_bytes = 4096u + static_cast<uint32_t>(p.nt) * 32u;  // pre-load MMA operands
         // the packed filters are bulk-copied into shared memory when they are whole 16-byte units and fit
-        const long long wraw = static_cast<long long>(s.m) * p.taps * cb;
+        const long long wraw = static_cast<long long>(s.m) * s.kh * s.kw * cb;
         bool placed = false;
         for (int copy_w : {1, 0}) {
           if (copy_w && (wraw % 16 != 0 || wraw > 96 * 1024)) continue;
@@ -178,6 +184,8 @@ win::WinArgs win_args(const WinPlan &plan, const ConvShape &s, const ConvParams 
     a.c_pad = plan.c_pad;
     a.groups = plan.groups;
     a.taps = plan.taps;
+    a.fold = plan.fold;
+    a.kwf = plan.kwf;
     a.ksteps = plan.ksteps;
     a.s = plan.s;
     a.sp = plan.sp;

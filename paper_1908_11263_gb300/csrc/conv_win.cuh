@@ -112,6 +112,8 @@ struct WinArgs {
     int shift;
     int n, h, w_, c, m, kh, kw, ph, pw, oh, ow;
     int c_pad, groups, taps, ksteps, s, sp, wh, npos;
+    int fold;                // kernel columns folded into K: a tap is a kernel row (INT-8, c * kw <= 16)
+    int kwf;                 // kernel columns as the MMAs see them (1 when folded)
     int cb;                  // packed bytes per input pixel
     int full_rows;
     int tiles_x, tiles_per_img, total_tiles;
@@ -345,6 +347,81 @@ __device__ __forceinline__ void converter_role(const WinArgs &a, uint8_t *smem, 
     }
 }
 
+// The folded layout (INT-8, kernel columns folded into K): position (row, col)
+// of the window holds the kw * c bytes of image pixels col .. col + kw - 1 of
+// its row, then zeros, staged as 16 fp16 values x - 128 in two K-chunk planes;
+// kernel row i of strip s reads the window i rows and 8s positions on.  The
+// raw stage holds whole image rows.  Activation 0 stands outside the image
+// (it stages as -128, like every padded value); the values past kw * c meet
+// zero weights.
+__device__ __forceinline__ void converter_fold(const WinArgs &a, uint8_t *smem, uint64_t *raw_full,
+                                               uint64_t *raw_empty, uint64_t *a_full, uint64_t *a_empty)
+{
+    const int tid = threadIdx.x;
+    int rs = 0, as = 0;
+    uint32_t r_ph = 0, a_ph = 0;
+    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+        const Geo g = geo_of(a, t);
+        const int r0 = row_lo(a, g), r1 = row_hi(a, g);
+        if (!mbar_wait_warp(&raw_full[rs], r_ph, a.status)) return;
+        if (!mbar_wait_warp(&a_empty[as], a_ph ^ 1u, a.status)) return;
+        const uint8_t *raw = smem + a.off_raw + rs * a.raw_bytes;
+        const uint32_t stage = smem_addr(smem + a.off_a + as * a.stage_bytes);
+#pragma unroll 1
+        for (int pos = tid; pos < a.npos; pos += 128) {
+            const int pr = fdiv(pos, a.fd_sp), pc = pos - pr * a.sp;
+            const int col = g.ix0 + pc;  // image column of the position's first pixel
+            // the span's pixels inside the image, [jlo, jhi); their bytes are contiguous in the row
+            const int jlo = max(0, -col), jhi = min(a.kw, a.w_ - col);
+            unsigned long long lo = 0ull, hi = 0ull;  // the 16 bytes, zero outside the image
+            if (pr >= r0 && pr < r1 && jhi > jlo) {
+                const uint8_t *row = raw + static_cast<uint32_t>(pr - r0) * a.raw_row_bytes;
+                // five aligned words from the first inside byte, funnel-shifted to it
+                const uint32_t off = static_cast<uint32_t>((col + jlo) * a.c);
+                const uint32_t *wp = reinterpret_cast<const uint32_t *>(row + (off & ~3u));
+                uint32_t q[5];
+#pragma unroll
+                for (int k = 0; k < 5; ++k) q[k] = wp[k];
+                const uint32_t sh = (off & 3u) * 8u;
+                lo = static_cast<unsigned long long>(__funnelshift_r(q[0], q[1], sh)) |
+                     static_cast<unsigned long long>(__funnelshift_r(q[1], q[2], sh)) << 32;
+                hi = static_cast<unsigned long long>(__funnelshift_r(q[2], q[3], sh)) |
+                     static_cast<unsigned long long>(__funnelshift_r(q[3], q[4], sh)) << 32;
+                // to byte jlo * c of the span (a 128-bit shift), then keep bytes [jlo * c, jhi * c)
+                const int s8 = jlo * a.c * 8;
+                if (s8 >= 64) {
+                    hi = lo << (s8 - 64);
+                    lo = 0ull;
+                } else if (s8 > 0) {
+                    hi = (hi << s8) | (lo >> (64 - s8));
+                    lo <<= s8;
+                }
+                const int b1 = jhi * a.c;  // bytes below b1 stay
+                const unsigned long long keep_lo = b1 >= 8 ? ~0ull : (1ull << (8 * b1)) - 1ull;
+                const unsigned long long keep_hi = b1 >= 16 ? ~0ull : b1 <= 8 ? 0ull : (1ull << (8 * (b1 - 8))) - 1ull;
+                lo &= keep_lo;
+                hi &= keep_hi;
+            }
+            uint32_t wd[4] = {static_cast<uint32_t>(lo), static_cast<uint32_t>(lo >> 32), static_cast<uint32_t>(hi),
+                              static_cast<uint32_t>(hi >> 32)};
+            const uint32_t pos16 = static_cast<uint32_t>(pos) * 16u;
+            sts128(stage + pos16, cvt_u8x8(make_uint2(wd[0], wd[1])));
+            sts128(stage + a.chunk_stride + pos16, cvt_u8x8(make_uint2(wd[2], wd[3])));
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(&a_full[as]);
+        mbar_arrive(&raw_empty[rs]);
+        if (++rs == a.raw_stages) {
+            rs = 0;
+            r_ph ^= 1u;
+        }
+        if (++as == a.a_stages) {
+            as = 0;
+            a_ph ^= 1u;
+        }
+    }
+}
+
 // ---------------------------------------------------------------- MMA issue (warp 12)
 
 __device__ __forceinline__ uint64_t desc_of(uint32_t lo, uint32_t hi)
@@ -413,11 +490,11 @@ __device__ __forceinline__ void mma_role(const WinArgs &a, uint8_t *smem, uint64
     const int nu = static_cast<int>(misc->nmma);
     // the common shapes with one exact chunk issue from unrolled code
     const int fixed = nch != kx ? 0
-                      : (a.kh == 3 && a.kw == 3 && a.ksteps == 2 && a.s == 2) ? 1
-                      : (a.kh == 3 && a.kw == 3 && a.ksteps == 1 && a.s == 2) ? 2
-                      : (a.kh == 5 && a.kw == 5 && a.ksteps == 2 && a.s == 2) ? 3
-                      : (a.kh == 5 && a.kw == 5 && a.ksteps == 2 && a.s == 1) ? 4
-                      : (a.kh == 3 && a.kw == 3 && a.ksteps == 4 && a.s == 2) ? 5
+                      : (a.kh == 3 && a.kwf == 3 && a.ksteps == 2 && a.s == 2) ? 1
+                      : (a.kh == 3 && a.kwf == 3 && a.ksteps == 1 && a.s == 2) ? 2
+                      : (a.kh == 5 && a.kwf == 5 && a.ksteps == 2 && a.s == 2) ? 3
+                      : (a.kh == 5 && a.kwf == 5 && a.ksteps == 2 && a.s == 1) ? 4
+                      : (a.kh == 3 && a.kwf == 3 && a.ksteps == 4 && a.s == 2) ? 5
                                                                                 : 0;
     for (int i = 0, t = blockIdx.x; t < a.total_tiles; ++i, t += gridDim.x) {
         const int as = i % a.a_stages, slot = i % nslots;
@@ -521,9 +598,11 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
     if (et == 0) misc->mask = ~0u;
     prep_sync();
     // item i: channel n = i % NT, tap i / NT; thread et takes items et, et + kPrepThreads, ...
-    const int cgroups = a.c * BITS / 8 / kGroupBytes;
+    // K-chunks holding filter values, and packed bytes of one tap of one filter (a kernel
+    // row's kw * c bytes when folded: they are contiguous in [m][kh][kw][c])
+    const int cgroups = a.fold ? a.groups : a.c * BITS / 8 / kGroupBytes;
     const int items = a.taps * NT;
-    const long long wrow = static_cast<long long>(a.c) * BITS / 8;  // packed bytes of one tap of one filter
+    const long long wrow = a.fold ? static_cast<long long>(a.kw) * a.c : static_cast<long long>(a.c) * BITS / 8;
     // the packed filters: the loader's shared-memory copy, or global memory
     const bool copied = a.wraw_bytes != 0;
     if (copied) mbar_wait_warp(w_full, 0, a.status);
@@ -537,7 +616,16 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
 #pragma unroll
             for (int gq = 0; gq < 8; ++gq) {
                 const bool has = i < items && n < a.m && gq < cgroups;
-                if (kGroupBytes == 8) {
+                if (BITS == 8 && a.fold) {
+                    // bytes gq * 8 .. + 7 of the row's kw * c (unaligned; zero past its end)
+                    uint32_t lo = 0, hi = 0;
+                    for (int k = 0; has && k < 8 && gq * 8 + k < wrow; ++k) {
+                        const uint32_t byte = src[gq * 8 + k];
+                        if (k < 4) lo |= byte << (8 * k);
+                        else hi |= byte << (8 * (k - 4));
+                    }
+                    raw[b][gq] = make_uint2(lo, hi);
+                } else if (kGroupBytes == 8) {
                     const uint2 *q = reinterpret_cast<const uint2 *>(src + gq * 8);
                     raw[b][gq] = !has ? make_uint2(0u, 0u) : copied ? *q : __ldg(q);
                 } else {
@@ -626,7 +714,7 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
         uint2 *tab = reinterpret_cast<uint2 *>(smem + a.off_mtab);
         const uint32_t kstep_a = 2u * (a.chunk_stride >> 4), kstep_b = 2u * NT;
         for (int c = 0; c < nj; ++c) {
-            const int tap = c * ct + jt, ti = tap / a.kw, tj = tap - ti * a.kw;
+            const int tap = c * ct + jt, ti = tap / a.kwf, tj = tap - ti * a.kwf;
             for (int s = 0; s < a.s; ++s, ++u)
                 tab[u] = make_uint2((static_cast<uint32_t>(ti * a.sp + tj) + kk * kstep_a + s * kCols) |
                                         (static_cast<uint32_t>((s * nch + c) * kx + kk % kx) * NT << 16),
@@ -1137,7 +1225,14 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     // prepares the filters and writes the image.
     const bool convolve = a.img_out == nullptr;
     if (warp < kConvWarps) {
-        if (convolve) converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
+        if (convolve) {
+            if constexpr (BITS == 8) {
+                if (a.fold) converter_fold(a, smem, raw_full, raw_empty, a_full, a_empty);
+                else converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
+            } else {
+                converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
+            }
+        }
     } else if (warp == kLoadWarp) {
         if (!a.img) load_filters(a, smem, w_full);
         if (convolve) {

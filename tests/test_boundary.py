@@ -151,8 +151,8 @@ def test_subbyte_layers_with_c_multiple_of_32_plan_e4m3_filters(lib):
 
 def test_window_kernel_selection_and_prepared_workspace(lib):
     """Tensor-core requests take the window kernel where its plan fits (the benchmark layer at
-    every Q, the CIFAR-shaped conv2 / conv3) and the general kernel elsewhere (C = 3, more than
-    128 output channels).  The window kernel's prepared workspace holds the image qconv_hwc_prepare
+    every Q, the CIFAR-shaped conv1 with its kernel columns folded into K, conv2 / conv3) and the
+    general kernel elsewhere (C * kw above 16 at C = 3, more than 128 output channels).  The window kernel's prepared workspace holds the image qconv_hwc_prepare
     builds: the filters as the B operand (taps x 4 K-chunks x 64 rows x 16 bytes), then the
     records (2 x 64 x 16 bytes + flags), the tap sums ((taps + 3) x 64 int32), the MMA table
     (2 strips x 9 taps x 2 k-steps x 8 bytes) and the pre-load operands (4 KB + 64 x 32 bytes)."""
@@ -160,7 +160,9 @@ def test_window_kernel_selection_and_prepared_workspace(lib):
         assert qnn.tc_kernel(desc(bits=bits)) == qnn.ALGO_TC_WINDOW
     assert qnn.tc_kernel(qnn.conv_desc(1024, 16, 16, 32, 32, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_WINDOW
     assert qnn.tc_kernel(qnn.conv_desc(1024, 8, 8, 32, 64, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_WINDOW
-    assert qnn.tc_kernel(qnn.conv_desc(1024, 32, 32, 3, 32, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_GENERAL
+    # C = 3: the kernel columns fold into K (kw * C = 15 values per position and kernel row)
+    assert qnn.tc_kernel(qnn.conv_desc(1024, 32, 32, 3, 32, 5, 5, 1, 2, 8, 10)) == qnn.ALGO_TC_WINDOW
+    assert qnn.tc_kernel(qnn.conv_desc(4, 32, 32, 3, 32, 7, 7, 1, 3, 8, 10)) == qnn.ALGO_TC_GENERAL  # 21 > 16
     assert qnn.tc_kernel(qnn.conv_desc(64, 14, 14, 256, 512, 1, 1, 1, 0, 8, 10)) == qnn.ALGO_TC_GENERAL
     assert qnn.tc_kernel(desc(algo=qnn.ALGO_TC_GENERAL)) == qnn.ALGO_TC_GENERAL
     assert qnn.tc_kernel(desc(stride=(2, 2))) == 0

@@ -5,6 +5,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_1908_11263_gb300 import inputs, qnn
 
 from gpu_util import conv_gpu, conv_oracle, dev, first_mismatch, layer_tensors, pack_gpu, tc_algos, to_dev
@@ -162,3 +163,50 @@ def test_prepared_graph_full_size(which):
         got = y.cpu().numpy().reshape(n, -1)
         exp = want if i % 2 == 0 else want[::-1]
         assert first_mismatch(got.reshape(-1), np.ascontiguousarray(exp).reshape(-1)) is None, (which, i)
+
+
+@pytest.mark.parametrize("shape", [
+    (2, 32, 32, 3, 32, 5, 5, 2),    # CIFAR conv1 shape: 15 of 16 values per kernel row
+    (2, 21, 32, 3, 16, 3, 3, 1),    # 9 values, a partial last tile row
+    (1, 16, 48, 5, 24, 3, 3, 1),    # 15 values, three tiles across
+    (2, 19, 16, 1, 8, 7, 7, 3),     # one channel, 7 wide
+    (1, 20, 32, 2, 40, 5, 5, 0),    # no padding
+    (3, 9, 16, 4, 32, 4, 4, 2),     # exactly 16 values, even kernel
+])
+@pytest.mark.parametrize("pool", [False, True])
+def test_folded_kernel_columns(shape, pool):
+    """Few input channels (C * kw <= 16, C not a multiple of 8): the window kernel folds the
+    kernel columns into K, so a staged position carries kw neighbouring pixels' channels and an
+    MMA covers one kernel row.  Every output byte equals the oracle's (and, with pool, the
+    oracle's conv followed by its 2x2 max-pool), on the folded window kernel and on the general
+    kernel, one-shot and prepared."""
+    n, h, w, c, m, k, _, p = shape
+    desc = qnn.conv_desc(n, h, w, c, m, k, k, 1, p, 8, 0)
+    assert qnn.tc_kernel(desc) == qnn.ALGO_TC_WINDOW
+    rng = np.random.default_rng(sum(shape) * 7 + int(pool))
+    x = rng.integers(0, 256, size=(n, h, w, c))
+    wt = rng.integers(-128, 128, size=(m, k, k, c))
+    kappa = rng.integers(1, 64, size=m).astype(np.int16)
+    bias = rng.integers(-4096, 4097, size=m).astype(np.int32)
+    shift = 12
+    lam = rng.integers(0, 256 << (shift - 1), size=m).astype(np.int32)
+    want = conv_oracle(x, wt, bias, kappa, lam, None, shift, 8, (1, 1), (p, p))
+    oh, ow = h + 2 * p - k + 1, w + 2 * p - k + 1
+    if pool:
+        want = oracle.maxpool(want, n, oh, ow, m, 2, 2, 8)
+    assert len(np.unique(want)) > 16, "outputs nearly constant: the check is weak"
+    xd, wd = to_dev(x.astype(np.uint8)), to_dev(wt.astype(np.int8))
+    kd, ld_, bd = to_dev(kappa), to_dev(lam), to_dev(bias)
+    for algo in (qnn.ALGO_TC_WINDOW, qnn.ALGO_TC_GENERAL):
+        if pool:
+            got = qnn.conv_hwc_pool2(xd, wd, kd, ld_, bias=bd, shift=shift, bits=8, pad=p, algo=algo)
+        else:
+            got = qnn.conv_hwc(xd, wd, kd, ld_, bias=bd, shift=shift, bits=8, stride=1, pad=p, algo=algo)
+        qnn.device_status()
+        got = got.cpu().numpy().reshape(-1)
+        assert first_mismatch(got, want) is None, (algo, first_mismatch(got, want))
+    if not pool:
+        prep = qnn.PreparedConv(wd, kd, ld_, n=n, h=h, wd=w, bias=bd, shift=shift, bits=8, stride=1, pad=p)
+        got = prep(xd).cpu().numpy().reshape(-1)
+        qnn.device_status()
+        assert first_mismatch(got, want) is None, ("prepared", first_mismatch(got, want))

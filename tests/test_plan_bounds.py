@@ -77,6 +77,9 @@ def test_window_plans_keep_every_access_in_bounds(tmp_path):
     for q, fmt in ((8, "fp16"), (4, "e4m3"), (2, "e4m3")):
         got = plans[f"512x16x16x32->64 k3x3 p1,1 q{q} pool0"]
         assert got.startswith(f"1 S=2 {fmt} nt=64") and got.endswith("full-rows"), (q, got)
-    # layers the window kernel leaves to the general kernel: C = 3, more than 128 output channels
-    assert plans["1024x32x32x3->32 k5x5 p2,2 q8 pool0"] == "0"
+    # CIFAR conv1 (C = 3): kernel columns folded into K, whole rows, one 16-value K-step per kernel row
+    got = plans["1024x32x32x3->32 k5x5 p2,2 q8 pool0"]
+    assert got.startswith("1 S=2 fp16 nt=32 sp=16 wh=20") and got.endswith("full-rows folded"), got
+    assert " folded" in text and text.count(" folded") >= 10
+    # a layer the window kernel leaves to the general kernel: more than 128 output channels
     assert plans["64x14x14x256->512 k1x1 p0,0 q8 pool0"] == "0"

@@ -64,9 +64,15 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
         std::printf("\n");
         return;
     }
-    std::printf(" S=%d %s nt=%d sp=%d wh=%d stages=%d/%d nch=%d..%d smem=%u wcopy=%u %s\n", p.s,
+    std::printf(" S=%d %s nt=%d sp=%d wh=%d stages=%d/%d nch=%d..%d smem=%u wcopy=%u %s%s\n", p.s,
                 p.fp8 ? "e4m3" : "fp16", p.nt, p.sp, p.wh, p.a_stages, p.raw_stages, p.nch_min, p.nch_max, p.smem_bytes,
-                p.wraw_bytes, p.full_rows ? "full-rows" : "row-segments");
+                p.wraw_bytes, p.full_rows ? "full-rows" : "row-segments", p.fold ? " folded" : "");
+    // folded plans: a tap is a kernel row, a position holds kw pixels' c channels
+    CHECK(p.fold == (bits == 8 && c % 8 != 0 && kw > 1 && c * kw <= 16), "fold rule");
+    CHECK(p.fold ? (p.taps == kh && p.kwf == 1 && p.groups == 2 && p.c_pad == 16 && p.full_rows &&
+                    p.sp == kCols * p.s)
+                 : (p.taps == kh * kw && p.kwf == kw && p.sp == kCols * p.s + kw - 1),
+          "fold layout");
     const long long cb = static_cast<long long>(c) * bits / 8;
     const int kch = p.fp8 ? 16 : 8, gbytes = kch * bits / 8;  // packed bytes of one K-chunk
     CHECK(gbytes == (bits == 8 ? 8 : 16 * bits / 8), "gbytes %d", gbytes);
@@ -81,7 +87,7 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
     CHECK(p.off_mtab % 8 == 0 && p.off_mtab + 8LL * p.s * p.taps * p.ksteps <= p.off_pre, "MMA table");
     CHECK(p.off_pre % 128 == 0 && p.off_pre + 4096LL + 32LL * p.nt <= p.off_wraw, "pre-load operands");
     CHECK(p.off_wraw % 16 == 0 && p.off_wraw + p.wraw_bytes <= p.off_bar, "filter copy");
-    if (p.wraw_bytes) CHECK(p.wraw_bytes == static_cast<long long>(m) * p.taps * cb && p.wraw_bytes % 16 == 0,
+    if (p.wraw_bytes) CHECK(p.wraw_bytes == static_cast<long long>(m) * kh * kw * cb && p.wraw_bytes % 16 == 0,
                             "filter copy size");
     CHECK(p.off_bar % 16 == 0 && p.off_bar + kBarBytes <= p.smem_bytes && p.smem_bytes <= kSmemLimit, "barriers");
     // the MMA issue table the filter preparation writes, for every chunk count the kernel
@@ -146,9 +152,16 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
     }
     CHECK(256 % p.nt == 0 && p.nt >= m, "prep channel per thread");
     // the filter-prep loads: the last K-chunk of the last channel inside the packed filters
-    CHECK((static_cast<long long>(m - 1) * p.taps + p.taps - 1) * cb + (c * bits / 8 / gbytes - 1) * gbytes + gbytes <=
-              static_cast<long long>(m) * p.taps * cb,
-          "prep loads");
+    // (folded: the bytes of a kernel row, kw * c of them, read one by one)
+    if (p.fold)
+        CHECK((static_cast<long long>(m - 1) * p.taps + p.taps - 1) * kw * c + kw * c <=
+                  static_cast<long long>(m) * kh * kw * c && kw * c <= 16,
+              "prep loads (folded)");
+    else
+        CHECK((static_cast<long long>(m - 1) * p.taps + p.taps - 1) * cb + (c * bits / 8 / gbytes - 1) * gbytes +
+                      gbytes <=
+                  static_cast<long long>(m) * p.taps * cb,
+              "prep loads");
     CHECK(p.taps * p.groups * p.nt * 16LL == p.b_bytes, "B size");
     // division used for window positions
     for (int pos = 0; pos < kMaxKP * kConvThreads; ++pos) CHECK(fdiv(pos, p.sp) == pos / p.sp, "fdiv sp %d", pos);
@@ -173,7 +186,46 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
                 CHECK(src >= 0 && src + seg <= x_bytes && src % 16 == 0, "copy source row %d", r);
                 CHECK(iy0 + r >= 0 && iy0 + r < h, "copied row inside the image");
             }
-            if (p.full_rows) CHECK(ix0 + c0 == 0 && ix0 + c1 == w, "whole rows");
+            if (p.full_rows && !p.fold) CHECK(ix0 + c0 == 0 && ix0 + c1 == w, "whole rows");
+            if (p.fold) {
+                // folded converter: whole image rows; a position inside the image in both
+                // directions reads five aligned words from its row's first byte, rounded
+                // down to 4; the words stay inside shared memory, the span inside the row
+                for (int pos = 0; pos < npos; ++pos) {
+                    const int r = fdiv(pos, p.sp), px = pos - r * p.sp, colx = ix0 + px;
+                    CHECK(2LL * p.chunk_stride <= p.stage_bytes && pos * 16LL + 16 <= p.chunk_stride, "folded store");
+                    if (r < r0 || r >= r1) {
+                        CHECK(iy0 + r < 0 || iy0 + r >= h, "folded row outside the image");
+                        continue;
+                    }
+                    CHECK(iy0 + r >= 0 && iy0 + r < h, "folded row inside the image");
+                    // the span's pixels inside the image, [jlo, jhi): their bytes from the first one on
+                    const int jlo = std::max(0, -colx), jhi = std::min(kw, w - colx);
+                    if (jhi <= jlo) continue;
+                    const long long off = static_cast<long long>(colx + jlo) * c;
+                    const long long word0 = static_cast<long long>(r - r0) * p.raw_row_bytes + (off & ~3LL);
+                    CHECK(off >= 0 && off + (jhi - jlo) * c <= static_cast<long long>(w) * c, "folded span inside the row");
+                    CHECK(jlo * c * 8 < 128 && jhi * c <= 16, "folded shift and mask");
+                    CHECK(p.raw_row_bytes % 4 == 0 &&
+                              p.off_raw + static_cast<long long>(p.raw_stages - 1) * p.raw_bytes + word0 + 20 <=
+                                  p.smem_bytes,
+                          "folded word loads");
+                }
+                for (int sj = 0; sj < p.s; ++sj)
+                    for (int i = 0; i < kh; ++i)
+                        for (int g = 0; g < kRows; ++g)
+                            for (int col = 0; col < kCols; ++col) {
+                                const int pos = i * p.sp + sj * kCols + g * p.sp + col;
+                                CHECK(pos >= 0 && pos < npos, "folded A row");
+                                const int r = pos / p.sp, px = pos % p.sp;
+                                const int oy = oy0 + g, ox = ox0 + sj * kCols + col;
+                                if (oy < s.oh && ox < s.ow)
+                                    CHECK(iy0 + r == oy - ph + i && ix0 + px == ox - pw, "folded A row pixels");
+                            }
+                for (int tap = 0; tap < p.taps; ++tap)
+                    CHECK((static_cast<long long>(tap) * p.groups + 2) * p.nt * 16 <= p.b_bytes, "folded B rows");
+                continue;
+            }
             // converter
             const int base_col = p.full_rows ? ix0 : -c0;
             for (int tid = 0; tid < kConvThreads; ++tid)
@@ -244,6 +296,8 @@ int main()
         {1, 16, 16, 32, 64, 3, 3, 1, 1, 8},     {2, 20, 36, 32, 64, 3, 3, 1, 1, 8},   {1, 17, 40, 64, 128, 7, 7, 3, 3, 8},
         {1, 9, 24, 128, 96, 3, 3, 1, 1, 4},     {1, 9, 24, 128, 96, 3, 3, 1, 1, 2},   {2, 3, 3, 32, 32, 3, 3, 1, 1, 8},
         {1, 16, 16, 64, 64, 3, 3, 1, 1, 8},     {1, 24, 40, 32, 32, 5, 5, 2, 2, 8},   {3, 18, 18, 16, 16, 3, 3, 0, 0, 8},
+        {2, 21, 32, 3, 16, 3, 3, 1, 1, 8},      {1, 16, 48, 5, 24, 3, 3, 1, 1, 8},    {2, 19, 16, 1, 8, 7, 7, 3, 3, 8},
+        {1, 20, 32, 2, 40, 5, 5, 0, 0, 8},      {3, 9, 16, 4, 32, 4, 4, 2, 1, 8},
     };
     for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 0);
     for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 1);
