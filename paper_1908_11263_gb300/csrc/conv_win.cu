@@ -34,7 +34,7 @@ WinPlan plan_conv_win(const ConvShape &s)
     p.kch = p.fp8 ? 16 : 8;
     // INT-8 with few channels (C * kw <= 16, C not a multiple of 8): a kernel row's kw * C
     // values of a position fill one 16-value K-step (two K-chunks)
-    p.fold = s.bits == 8 && s.c % 8 != 0 && s.kw > 1 && s.c * s.kw <= 16;
+    p.fold = s.bits == 8 && s.c % 8 != 0 && s.kw > 1 && s.c * s.kw <= 16 && s.m <= 64;
     p.kwf = p.fold ? 1 : s.kw;
     // INT-8 in fp16 (whole 8-channel chunks), INT-4 / INT-2 in e4m3 (whole 32-channel pairs)
     if (!p.fold && (s.bits == 8 ? (s.c % 8 != 0) : (s.c % 32 != 0))) return p;

@@ -585,7 +585,7 @@ __device__ __forceinline__ uint4 filter_chunk(uint2 v, int &pos, int &neg, int &
 // the chunk count they allow, the MMA issue table, the pre-load operands and
 // the slot layout.  The per-channel sums of positive and negative weights
 // stay in shared memory for the compression records.
-template <int BITS, int NT>
+template <int BITS, int NT, bool FOLD>
 __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem, Misc *misc, uint64_t *w_full)
 {
     constexpr int kGroupBytes = BITS == 8 ? 8 : 16 * BITS / 8;
@@ -600,9 +600,9 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
     // item i: channel n = i % NT, tap i / NT; thread et takes items et, et + kPrepThreads, ...
     // K-chunks holding filter values, and packed bytes of one tap of one filter (a kernel
     // row's kw * c bytes when folded: they are contiguous in [m][kh][kw][c])
-    const int cgroups = a.fold ? a.groups : a.c * BITS / 8 / kGroupBytes;
+    const int cgroups = FOLD ? a.groups : a.c * BITS / 8 / kGroupBytes;
     const int items = a.taps * NT;
-    const long long wrow = a.fold ? static_cast<long long>(a.kw) * a.c : static_cast<long long>(a.c) * BITS / 8;
+    const long long wrow = FOLD ? static_cast<long long>(a.kw) * a.c : static_cast<long long>(a.c) * BITS / 8;
     // the packed filters: the loader's shared-memory copy, or global memory
     const bool copied = a.wraw_bytes != 0;
     if (copied) mbar_wait_warp(w_full, 0, a.status);
@@ -616,7 +616,7 @@ __device__ __forceinline__ void prepare_filters(const WinArgs &a, uint8_t *smem,
 #pragma unroll
             for (int gq = 0; gq < 8; ++gq) {
                 const bool has = i < items && n < a.m && gq < cgroups;
-                if (BITS == 8 && a.fold) {
+                if constexpr (BITS == 8 && FOLD) {
                     // bytes gq * 8 .. + 7 of the row's kw * c (unaligned; zero past its end)
                     uint32_t lo = 0, hi = 0;
                     for (int k = 0; has && k < 8 && gq * 8 + k < wrow; ++k) {
@@ -1166,7 +1166,7 @@ __device__ __forceinline__ void epilogue_role(const WinArgs &a, uint8_t *smem, u
 
 // ---------------------------------------------------------------- the kernel
 
-template <int BITS, int NT, bool POOL>
+template <int BITS, int NT, bool POOL, bool FOLD>
 __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
 {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -1226,12 +1226,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
     const bool convolve = a.img_out == nullptr;
     if (warp < kConvWarps) {
         if (convolve) {
-            if constexpr (BITS == 8) {
-                if (a.fold) converter_fold(a, smem, raw_full, raw_empty, a_full, a_empty);
-                else converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
-            } else {
-                converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
-            }
+            if constexpr (BITS == 8 && FOLD) converter_fold(a, smem, raw_full, raw_empty, a_full, a_empty);
+            else converter_role<BITS>(a, smem, raw_full, raw_empty, a_full, a_empty);
         }
     } else if (warp == kLoadWarp) {
         if (!a.img) load_filters(a, smem, w_full);
@@ -1244,7 +1240,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_win_kernel(const WinArgs a)
         if (a.img) {
             image_ready<NT>(a, smem, misc, w_full);
         } else {
-            prepare_filters<BITS, NT>(a, smem, misc, w_full);
+            prepare_filters<BITS, NT, FOLD>(a, smem, misc, w_full);
         }
         if (warp == kMmaWarp) {
             if (convolve) mma_role<NT, BITS != 8>(a, smem, a_full, a_empty, acc_full, acc_empty, done, misc);

@@ -13,13 +13,13 @@
 namespace qnn {
 namespace {
 
-template <int BITS, int NT, bool POOL>
+template <int BITS, int NT, bool POOL, bool FOLD = false>
 cudaError_t launch_one(const win::WinArgs &a, int grid, uint32_t smem, cudaStream_t st)
 {
     // the opt-in shared-memory limit is raised once per device, outside any stream capture
     static std::mutex mu;
     static bool raised[64] = {};
-    auto kern = win::conv_win_kernel<BITS, NT, POOL>;
+    auto kern = win::conv_win_kernel<BITS, NT, POOL, FOLD>;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -53,6 +53,18 @@ template <>
 cudaError_t launch_win_bits<QNN_WIN_BITS>(const win::WinArgs &a, int nt, int grid, uint32_t smem, cudaStream_t st)
 {
     constexpr int B = QNN_WIN_BITS;
+#if QNN_WIN_BITS == 8
+    // folded plans (few input channels) have their own instantiations, at most 64 filters
+    if (a.fold) {
+        switch (nt) {
+            case 32: return a.pool ? launch_one<B, 32, true, true>(a, grid, smem, st)
+                                   : launch_one<B, 32, false, true>(a, grid, smem, st);
+            case 64: return a.pool ? launch_one<B, 64, true, true>(a, grid, smem, st)
+                                   : launch_one<B, 64, false, true>(a, grid, smem, st);
+            default: return cudaErrorInvalidValue;
+        }
+    }
+#endif
     switch (nt) {
         case 32: return a.pool ? launch_one<B, 32, true>(a, grid, smem, st) : launch_one<B, 32, false>(a, grid, smem, st);
         case 64: return a.pool ? launch_one<B, 64, true>(a, grid, smem, st) : launch_one<B, 64, false>(a, grid, smem, st);

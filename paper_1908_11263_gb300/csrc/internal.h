@@ -84,7 +84,7 @@ struct WinPlan {
     int kch;              // channels per 16-byte K-chunk: 8 (fp16) or 16 (e4m3)
     int c_pad;            // channels per tap rounded up to two K-chunks
     int groups;           // K-chunks per tap (c_pad / kch)
-    int fold;             // kernel columns folded into K (INT-8, C not a multiple of 8, C * kw <= 16):
+    int fold;             // kernel columns folded into K (INT-8, C not a multiple of 8, C * kw <= 16, m <= 64):
                           // a staged position holds its kw horizontal neighbours' channels, one MMA "tap"
                           // per kernel row
     int kwf;              // kernel columns as the MMAs see them: kw, or 1 when folded

@@ -68,7 +68,7 @@ static void check(int n, int h, int w, int c, int m, int kh, int kw, int ph, int
                 p.fp8 ? "e4m3" : "fp16", p.nt, p.sp, p.wh, p.a_stages, p.raw_stages, p.nch_min, p.nch_max, p.smem_bytes,
                 p.wraw_bytes, p.full_rows ? "full-rows" : "row-segments", p.fold ? " folded" : "");
     // folded plans: a tap is a kernel row, a position holds kw pixels' c channels
-    CHECK(p.fold == (bits == 8 && c % 8 != 0 && kw > 1 && c * kw <= 16), "fold rule");
+    CHECK(p.fold == (bits == 8 && c % 8 != 0 && kw > 1 && c * kw <= 16 && m <= 64), "fold rule");
     CHECK(p.fold ? (p.taps == kh && p.kwf == 1 && p.groups == 2 && p.c_pad == 16 && p.full_rows &&
                     p.sp == kCols * p.s)
                  : (p.taps == kh * kw && p.kwf == kw && p.sp == kCols * p.s + kw - 1),
