@@ -58,7 +58,7 @@ METRIC = "qconv_hwc GMAC/s (16x16x32 -> 64, 3x3, stride 1, pad 1, INT-8, batch 5
 
 PROFILE = os.path.join(ROOT, "profiles", "conv_win_kernel_conv3x3_16x16x32to64_int8_n512.md")
 KERNEL_SOURCES = ("conv_win.cuh", "conv_win_inst.cuh", "conv_common.cuh", "device.cuh", "internal.h")
-KERNEL_NAME = "conv_win_kernel<8,64,false>"
+KERNEL_NAME = "conv_win_kernel<8,64,false,false>"
 
 
 def measured_traffic():
