@@ -556,27 +556,43 @@ __device__ __forceinline__ uint4 filter_chunk(uint2 v, int &pos, int &neg, int &
         abs += all - 2 * ng;
         // byte b ^ 0x80 is the weight plus 128 as an unsigned byte: the activation encoding gives the weight
         return cvt_u8x8(make_uint2(v.x ^ 0x80808080u, v.y ^ 0x80808080u));
-    } else {
-    uint8_t e[16];
+    } else if constexpr (BITS == 4) {
+        // 16 signed nibbles: sums from nibble sums (a negative nibble n stands for n - 16),
+        // e4m3 codes by two prmt lookups (0..7 directly, 8..15 by magnitude 16 - n) plus the sign
+        int all = 0, ng = 0;
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-        constexpr int per = 32 / BITS;  // values per 32-bit word
-        const uint32_t word = k / per == 0 ? v.x : v.y;
-        const int f = (word >> ((k % per) * BITS)) & ((1 << BITS) - 1);
-        const int wv = f >= (1 << (BITS - 1)) ? f - (1 << BITS) : f;
-        pos += max(wv, 0);
-        neg += min(wv, 0);
-        abs += wv < 0 ? -wv : wv;
-        // INT-2 slots follow the converter's word order (even channels, then odd, per half)
-        const int slot = BITS == 4 ? k : (k & 8) + (k & 1) * 4 + ((k & 7) >> 1);
-        e[slot] = e4m3_of_int(wv);
-    }
-    uint4 r;
-    r.x = e[0] | e[1] << 8 | e[2] << 16 | static_cast<uint32_t>(e[3]) << 24;
-    r.y = e[4] | e[5] << 8 | e[6] << 16 | static_cast<uint32_t>(e[7]) << 24;
-    r.z = e[8] | e[9] << 8 | e[10] << 16 | static_cast<uint32_t>(e[11]) << 24;
-    r.w = e[12] | e[13] << 8 | e[14] << 16 | static_cast<uint32_t>(e[15]) << 24;
-    return r;
+        for (int h = 0; h < 2; ++h) {
+            const uint32_t x = h ? v.y : v.x;
+            const int nneg = __popc(x & 0x88888888u);
+            const uint32_t xm = x & (((x & 0x88888888u) >> 3) * 0xFu);  // the negative nibbles
+            all += __dp4a(static_cast<int>((x & 0x0F0F0F0Fu) + ((x >> 4) & 0x0F0F0F0Fu)), 0x01010101, 0) - 16 * nneg;
+            ng += __dp4a(static_cast<int>((xm & 0x0F0F0F0Fu) + ((xm >> 4) & 0x0F0F0F0Fu)), 0x01010101, 0) - 16 * nneg;
+        }
+        neg += ng;
+        pos += all - ng;
+        abs += all - 2 * ng;
+        auto code4 = [](uint32_t q) {  // the low 16 bits of q: four signed nibbles -> four e4m3 bytes
+            const uint32_t sgn = ((q & 0x8u) << 4) | ((q & 0x80u) << 8) | ((q & 0x800u) << 12) | ((q & 0x8000u) << 16);
+            return prmt(0x44403800u, 0x4E4C4A48u, q) | prmt(0x4A4C4E50u, 0x38404448u, q ^ 0x8888u) | sgn;
+        };
+        return make_uint4(code4(v.x), code4(v.x >> 16), code4(v.y), code4(v.y >> 16));
+    } else {
+        // 16 signed crumbs (one word): sums from crumb sums (a negative crumb c stands for
+        // c - 4), e4m3 codes by one 4-entry prmt lookup, in the converter's word order
+        // (even channels, then odd, per half)
+        const uint32_t x = v.x;
+        const int nneg = __popc(x & 0xAAAAAAAAu);
+        const uint32_t xm = x & (((x & 0xAAAAAAAAu) >> 1) * 0x3u);  // the negative crumbs
+        const uint32_t c = (x & 0x33333333u) + ((x >> 2) & 0x33333333u);
+        const uint32_t cm = (xm & 0x33333333u) + ((xm >> 2) & 0x33333333u);
+        const int all = __dp4a(static_cast<int>((c & 0x0F0F0F0Fu) + ((c >> 4) & 0x0F0F0F0Fu)), 0x01010101, 0) - 4 * nneg;
+        const int ng = __dp4a(static_cast<int>((cm & 0x0F0F0F0Fu) + ((cm >> 4) & 0x0F0F0F0Fu)), 0x01010101, 0) - 4 * nneg;
+        neg += ng;
+        pos += all - ng;
+        abs += all - 2 * ng;
+        constexpr uint32_t kCode = 0xB8C03800u;  // e4m3 of 0, 1, -2, -1 (crumbs 0..3)
+        const uint32_t ev = x & 0x33333333u, od = (x >> 2) & 0x33333333u;
+        return make_uint4(prmt(kCode, 0u, ev), prmt(kCode, 0u, od), prmt(kCode, 0u, ev >> 16), prmt(kCode, 0u, od >> 16));
     }
 }
 
