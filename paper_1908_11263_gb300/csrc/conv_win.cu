@@ -1,5 +1,6 @@
-// Host side of the window kernel (conv_win.cuh): the planner, the launch and
-// the prepared-workspace layout.
+// Host side of the window kernel (conv_win.cuh): the planner, the launches
+// (convolving, and the one-block launch that writes a prepared image) and the
+// prepared-workspace layout.
 #include <algorithm>
 
 #include "conv_win.cuh"

@@ -16,6 +16,9 @@
 // 8-row core-matrix groups are the sixteen output rows, sp positions apart.
 // One shared-memory descriptor per MMA, no im2col buffer and no shifted
 // copies (Eq. 7: neighbouring output pixels read neighbouring window pixels).
+// With few input channels (INT-8, c * kw <= 16) the kernel columns fold into
+// K instead: a staged position holds the c channels of kw neighbouring pixels,
+// the window is 8S positions wide and each MMA covers one kernel row.
 //
 // Exactness on fp16 / e4m3 tensor cores (there is no integer tcgen05 MMA on
 // this GPU).  INT-8 activations are staged as x - 128 in fp16, INT-4 / INT-2
@@ -31,10 +34,14 @@
 // nch_max, always valid).
 //
 // Filters in the kernel.  The loader first bulk-copies the packed filters and
-// the first windows' input rows; meanwhile the whole block turns the filters
-// into the B operand (K-major core matrices), derives the per-channel
-// compression records, the chunk count and the MMA issue order, all in shared
-// memory.  So one qconv_hwc call is one launch and needs no workspace.
+// the first windows' input rows; meanwhile the epilogue warps and the MMA warp
+// turn the filters into the B operand (K-major core matrices) and derive the
+// chunk count and the MMA issue order, and the epilogue warps the per-channel
+// compression records, all in shared memory, while the converters stage the
+// first windows.  So one qconv_hwc call is one launch and needs no workspace.
+// qconv_hwc_prepare runs the same preparation once, in a one-block launch
+// that writes the resulting shared-memory image to a workspace, and each
+// qconv_hwc_run launch copies that image instead of preparing.
 //
 // Warp roles after that (one persistent CTA per SM, 14 warps):
 //   warps 0-3   converters: raw window -> staged operand, every position

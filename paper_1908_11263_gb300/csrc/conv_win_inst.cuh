@@ -1,5 +1,6 @@
 // Instantiations of the window kernel for one bit width (QNN_WIN_BITS), by
-// output-channel tile and fused pool.  Included once by each conv_win_q*.cu.
+// output-channel tile, fused pool and (INT-8, at most 64 filters) folded
+// kernel columns.  Included once by each conv_win_q*.cu.
 #pragma once
 
 #include <mutex>
