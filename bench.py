@@ -761,14 +761,31 @@ def run_cifar_pipeline(layers, layer_tensors, graph_time, stream, dev):
             a = bufs[2 * li + 1]
         qnn.linear(a.view(n, -1), fw, fb, out=out_fused, stream=stream)
 
+    # the filters of an inference network prepared once, at set-up (qconv_hwc_prepare); each step is
+    # then one qconv_hwc_pool2_run launch per layer and the FC layer
+    preps = [qnn.PreparedConv(t["w"], t["kappa"], t["lam"], n=n, h=layer.h, wd=layer.w, bias=t["bias"],
+                              shift=t["shift"], bits=8, stride=1, pad=layer.pad, stream=stream)
+             for t, (_, layer, _, _) in zip(tensors, layers)]
+    out_prepared = torch.empty_like(out)
+
+    def net_prepared(_):
+        a = xin
+        for li, prep in enumerate(preps):
+            prep.pool2(a, out=bufs[2 * li + 1], stream=stream)
+            a = bufs[2 * li + 1]
+        qnn.linear(a.view(n, -1), fw, fb, out=out_prepared, stream=stream)
+
     macs = sum(layer.macs for (_, layer, _, _) in layers) + n * 1024 * 10
     with torch.cuda.stream(stream):
         net(0)
         net_fused(0)
+        net_prepared(0)
     torch.cuda.synchronize(dev)
-    same = bool(torch.equal(out, out_fused))
+    same = bool(torch.equal(out, out_fused)) and bool(torch.equal(out, out_prepared))
     for fn, name in ((net, "cifar_pipeline_n1024 (3 conv + 3 pool + FC, one graph)"),
-                     (net_fused, "cifar_pipeline_fused_n1024 (3 fused conv+pool + FC, one graph)")):
+                     (net_fused, "cifar_pipeline_fused_n1024 (3 fused conv+pool + FC, one graph)"),
+                     (net_prepared, "cifar_pipeline_fused_prepared_n1024 (filters prepared once; 3 fused conv+pool "
+                                    "runs + FC, one graph)")):
         t_net = graph_time(fn, 20, 5)
         qnn.device_status(stream)
         print(json.dumps({"sweep": "3", "layer": name, "macs": macs, "gmacs_call": round(macs / t_net / 1e9, 1),

@@ -178,6 +178,20 @@ qnn_status qconv_hwc_pool2(const qnn_conv_desc *d, const void *x, const void *w,
                            void *workspace, size_t workspace_bytes, void *stream);
 
 /*
+ * qconv_hwc_pool2_run: qconv_hwc_pool2() on filters prepared with
+ * qconv_hwc_prepare() for the same descriptor: the fused convolution,
+ * compression and 2x2/2 max-pool, one launch that reads x, the workspace and
+ * writes the pooled y ([n][oh/2][ow/2][m], packed Q-bit, 16-byte aligned).
+ * Only where qconv_hwc_algo() reports the window tensor-core kernel
+ * (qconv_hwc_tc_kernel() == QNN_ALGO_TC_WINDOW); QNN_EUNSUPPORTED otherwise,
+ * QNN_EINVAL when oh or ow is below 2, QNN_EWORKSPACE for a workspace below
+ * qconv_hwc_workspace_size() or not 256-byte aligned.  The workspace rules of
+ * qconv_hwc_run() apply (it is read before the wait on the previous kernel).
+ */
+qnn_status qconv_hwc_pool2_run(const qnn_conv_desc *d, const void *x, void *y, const void *workspace,
+                               size_t workspace_bytes, void *stream);
+
+/*
  * Quantized convolution with staircase compression (Sec. III-A, Eq. 4), the
  * paper's compression for INT-4 and INT-2 outputs:
  *

@@ -332,6 +332,28 @@ qnn_status qconv_hwc_pool2(const qnn_conv_desc *d, const void *x, const void *w,
     return from_cuda(e);
 }
 
+qnn_status qconv_hwc_pool2_run(const qnn_conv_desc *d, const void *x, void *y, const void *workspace,
+                               size_t workspace_bytes, void *stream)
+{
+    ConvShape s;
+    qnn_status st = check_conv(d, &s);
+    if (st != QNN_OK) return st;
+    if (s.oh < 2 || s.ow < 2) return QNN_EINVAL;  // no pooled pixel
+    if (s.n > 0 && (!x || !y)) return QNN_EINVAL;
+    if (!aligned(x, 16) || !aligned(y, 16)) return QNN_EALIGN;
+    // the kernel and plan qconv_hwc_prepare chose for this descriptor (the window
+    // planner's layout does not depend on the fused pool)
+    const Choice c = choose(d, s);
+    if (c.kernel < 0) return static_cast<qnn_status>(-c.kernel);
+    if (c.kernel != kWindow) return QNN_EUNSUPPORTED;
+    if (!workspace || workspace_bytes < c.wplan.img_bytes || !aligned(workspace, 256)) return QNN_EWORKSPACE;
+    s.pool = 1;
+    ConvParams p{};
+    p.x = static_cast<const uint8_t *>(x);
+    p.y = static_cast<uint8_t *>(y);
+    return from_cuda(launch_conv_win(c.wplan, s, p, static_cast<cudaStream_t>(stream), workspace));
+}
+
 qnn_status qconv_hwc_thresholds(const qnn_conv_desc *d, const void *x, const void *w, const int32_t *thresholds,
                                 void *y, void *workspace, size_t workspace_bytes, void *stream)
 {

@@ -26,7 +26,7 @@ ALGO_AUTO, ALGO_DIRECT, ALGO_TENSORCORE, ALGO_TC_WINDOW, ALGO_TC_GENERAL = 0, 1,
 
 EXPORTED = ("qconv_hwc_workspace_size", "qconv_hwc", "qconv_hwc_prepare", "qconv_hwc_run", "qconv_hwc_algo", "qlinear", "qmaxpool", "pack_subbyte",
             "unpack_subbyte", "qnn_device_status", "qnn_status_string", "qnn_version", "qconv_hwc_noalloc",
-            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary", "qconv_hwc_pool2",
+            "qnn_selftest_wait_timeout", "qconv_hwc_thresholds", "qconv_hwc_binary", "qconv_hwc_pool2", "qconv_hwc_pool2_run",
             "qconv_hwc_mma_operand_bits", "qconv_hwc_tc_kernel")
 
 
@@ -73,6 +73,8 @@ def load(build_if_missing: bool = False):
         lib.qconv_hwc_prepare.restype = I32
         lib.qconv_hwc_run.argtypes = [DP, P, P, P, SZ, P]
         lib.qconv_hwc_run.restype = I32
+        lib.qconv_hwc_pool2_run.argtypes = [DP, P, P, P, SZ, P]
+        lib.qconv_hwc_pool2_run.restype = I32
         lib.qconv_hwc_algo.argtypes = [DP]
         lib.qconv_hwc_noalloc.argtypes = [DP, P, P, P, P, P, P, P, P]
         lib.qconv_hwc_thresholds.argtypes = [DP, P, P, P, P, P, SZ, P]
@@ -383,6 +385,18 @@ class PreparedConv:
         st = load().qconv_hwc_run(ctypes.byref(self.desc), _ptr(x), _ptr(out), _ptr(self.workspace),
                                   ctypes.c_size_t(self.nbytes), _stream(stream))
         _check(st, "qconv_hwc_run")
+        return out
+
+    def pool2(self, x, out=None, stream=None):
+        """The convolution with its 2x2 stride-2 max-pool fused (qconv_hwc_pool2_run); returns
+        uint8 [n, oh // 2, ow // 2, m*Q/8]."""
+        _dev(x, torch.uint8, "x")
+        if out is None:
+            n, _, _, mb = self.out_shape
+            out = torch.empty((n, self.oh // 2, self.ow // 2, mb), dtype=torch.uint8, device=x.device)
+        st = load().qconv_hwc_pool2_run(ctypes.byref(self.desc), _ptr(x), _ptr(out), _ptr(self.workspace),
+                                        ctypes.c_size_t(self.nbytes), _stream(stream))
+        _check(st, "qconv_hwc_pool2_run")
         return out
 
 

@@ -141,10 +141,62 @@ def test_conv_pool2_cifar_chain_batch1024():
     np.testing.assert_array_equal(yd.cpu().numpy(), yo)
 
 
+@pytest.mark.gpu
+def test_conv_pool2_prepared_cifar_chain_batch1024():
+    """The CIFAR-10-shaped network of Sec. V-E at batch 1024 on prepared filters: each layer's
+    filters prepared once (qconv_hwc_prepare), then every convolution with its 2x2 max-pool
+    fused run from the prepared workspace (qconv_hwc_pool2_run), chained on the device, twice
+    over the same input (the workspaces are reused), then the fully connected layer.  Every
+    pooled activation and the FC outputs equal the oracle's chain."""
+    from paper_1908_11263_gb300 import inputs
+    n = 1024
+    x = inputs.cifar_input(n)
+    x0 = to_dev(x.astype(np.uint8))
+    layers = inputs.cifar_layers(n)
+    preps, want = [], []
+    xo = x.astype(np.uint8).reshape(-1)
+    for key, layer, wl, lid in layers:
+        ld = inputs.make_layer(key, layer, wl, lid, x=np.zeros(1))
+        preps.append(qnn.PreparedConv(to_dev(ld.w), to_dev(ld.kappa, torch.int16), to_dev(ld.lam, torch.int32),
+                                      n=n, h=layer.h, wd=layer.w, bias=to_dev(ld.bias, torch.int32), shift=ld.shift,
+                                      bits=8, stride=1, pad=layer.pad))
+        xo = oracle.conv_hwc_pool2(xo, ld.w.reshape(-1).view(np.uint8), layer.shape(), ld.bias, ld.kappa, ld.lam,
+                                   shift=ld.shift, nthreads=THREADS)
+        want.append(xo)
+    wfc, bfc = inputs.cifar_fc()
+    want_fc = oracle.linear(want[-1].reshape(n, -1), wfc, bfc)
+    for trial in range(2):
+        xd = x0
+        for (key, _, _, _), prep, yo in zip(layers, preps, want):
+            xd = prep.pool2(xd)
+            qnn.device_status()
+            got = xd.cpu().numpy().reshape(-1)
+            assert first_mismatch(got, yo) is None, (trial, key, first_mismatch(got, yo))
+        yd = qnn.linear(xd.view(n, -1), to_dev(wfc), to_dev(bfc))
+        np.testing.assert_array_equal(yd.cpu().numpy(), want_fc)
+
+
 @pytest.fixture(scope="module")
 def lib():
     qbuild.build()
     return qnn.load()
+
+
+def test_conv_pool2_run_rejects_what_it_cannot_run(lib):
+    """qconv_hwc_pool2_run: argument checks only (no CUDA call is reached)."""
+    P = ctypes.c_void_p
+
+    def status(d, ws=FAKE, nbytes=1 << 30, x=FAKE):
+        return lib.qconv_hwc_pool2_run(ctypes.byref(d), P(x), P(FAKE), P(ws), ctypes.c_size_t(nbytes), None)
+
+    ok = qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 1, 1, 8, 10)
+    assert status(qnn.conv_desc(1, 8, 8, 32, 32, 3, 3, 2, 1, 8, 10)) == qnn.QNN_EUNSUPPORTED  # stride 2
+    assert status(qnn.conv_desc(64, 14, 14, 256, 512, 1, 1, 1, 0, 8, 10)) == qnn.QNN_EUNSUPPORTED  # general kernel
+    assert status(qnn.conv_desc(1, 2, 2, 32, 32, 3, 3, 1, 0, 8, 10)) == qnn.QNN_EINVAL  # 0 x 0 output
+    assert status(ok, x=FAKE + 2) == qnn.QNN_EALIGN
+    assert status(ok, ws=None) == qnn.QNN_EWORKSPACE
+    assert status(ok, nbytes=256) == qnn.QNN_EWORKSPACE
+    assert status(ok, ws=FAKE + 16) == qnn.QNN_EWORKSPACE
 
 
 def test_conv_pool2_rejects_what_it_cannot_run(lib):
