@@ -16,7 +16,9 @@
 //   - exactness: the planner's worst-case chunk count keeps every chunk within
 //     2^22, and its even tap split has no empty chunk;
 //   - the reciprocal division the kernel uses for tile and window indices.
-// Prints one line per plan and "fails=N"; exits non-zero on any failure.
+// The shapes are the parity tests' and the workloads', then 300 seeded random
+// ones across the planner's range.  Prints one line per plan and "fails=N";
+// exits non-zero on any failure.
 #include <algorithm>
 #include <cstdint>
 #include <cstdio>
@@ -301,6 +303,23 @@ int main()
     };
     for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 0);
     for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 1);
+    // seeded random shapes across the planner's range (whatever it accepts is checked)
+    unsigned long long rng = 0x5EEDB0D5ull;
+    auto next = [&](int lo, int hi) {  // uniform in [lo, hi]
+        rng = rng * 6364136223846793005ull + 1442695040888963407ull;
+        return lo + static_cast<int>((rng >> 33) % static_cast<unsigned long long>(hi - lo + 1));
+    };
+    for (int i = 0; i < 300; ++i) {
+        static const int kBits[4] = {8, 8, 4, 2};
+        const int bits = kBits[next(0, 3)];
+        const int per = 8 / bits;
+        const int c = bits == 8 ? (next(0, 3) == 0 ? next(1, 7) : 8 * next(1, 8)) : 32 * next(1, bits == 4 ? 4 : 8);
+        const int m = per * next(1, 128 / per);
+        const int kh = next(1, 7), kw = next(1, 7);
+        const int ph = next(0, kh / 2), pw = next(0, kw / 2);
+        const int h = next(std::max(1, kh - 2 * ph), 40), w = next(std::max(1, kw - 2 * pw), 48);
+        check(next(1, 3), h, w, c, m, kh, kw, ph, pw, bits, next(0, 1));
+    }
     std::printf("fails=%d\n", fails);
     return fails ? 1 : 0;
 }
