@@ -210,3 +210,60 @@ def test_folded_kernel_columns(shape, pool):
         got = prep(xd).cpu().numpy().reshape(-1)
         qnn.device_status()
         assert first_mismatch(got, want) is None, ("prepared", first_mismatch(got, want))
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_shapes(seed):
+    """Seeded random layers across the window planner's range (bit width, channels including the
+    folded few-channel case, filters, kernel, padding, image size, fused pool): every tensor-core
+    kernel that takes the layer equals the oracle byte for byte."""
+    rng = np.random.default_rng(1000 + seed)
+    bits = int(rng.choice([8, 8, 4, 2]))
+    per = 8 // bits
+    if bits == 8:
+        c = int(rng.integers(1, 6)) if rng.integers(0, 3) == 0 else 8 * int(rng.integers(1, 9))
+    else:
+        c = 32 * int(rng.integers(1, 3))
+    m = per * int(rng.integers(1, 96 // per + 1))
+    kh, kw = int(rng.integers(1, 6)), int(rng.integers(1, 6))
+    ph, pw = int(rng.integers(0, kh // 2 + 1)), int(rng.integers(0, kw // 2 + 1))
+    n = int(rng.integers(1, 4))
+    h = int(rng.integers(max(2, kh - 2 * ph + 1), 30))
+    w = int(rng.integers(max(2, kw - 2 * pw + 1), 36))
+    pool = bool(rng.integers(0, 2))
+    desc = qnn.conv_desc(n, h, w, c, m, kh, kw, 1, (ph, pw), bits, 0)
+    algos = tc_algos(n, h, w, c, m, kh, kw, (1, 1), (ph, pw), bits)
+    if not algos:
+        pytest.skip("no tensor-core kernel takes this layer")
+    top = (1 << bits) - 1
+    x = rng.integers(0, top + 1, size=(n, h, w, c))
+    wt = rng.integers(-(1 << (bits - 1)), 1 << (bits - 1), size=(m, kh, kw, c))
+    taps = kh * kw * c
+    shift = {8: 12, 4: 8, 2: 6}[bits]
+    kappa = rng.integers(1, 64, size=m).astype(np.int16)
+    bias = rng.integers(-(taps * top), taps * top + 1, size=m).astype(np.int32)
+    lam = rng.integers(0, (top + 1) << shift, size=m).astype(np.int32)
+    oh, ow = h + 2 * ph - kh + 1, w + 2 * pw - kw + 1
+    want = conv_oracle(x, wt, bias, kappa, lam, None, shift, bits, (1, 1), (ph, pw))
+    if pool:
+        if oh < 2 or ow < 2:
+            pytest.skip("no pooled pixel")
+        want = oracle.maxpool(want, n, oh, ow, m, 2, 2, bits)
+    xd = pack_gpu(x, bits).view(n, h, w, c // per)
+    wd = pack_gpu(wt, bits).view(m, kh, kw, c // per)
+    if bits == 8:
+        wd = wd.view(torch.int8)
+    kd, ld_, bd = to_dev(kappa), to_dev(lam), to_dev(bias)
+    for algo in algos:
+        if pool:
+            got = qnn.conv_hwc_pool2(xd, wd, kd, ld_, bias=bd, shift=shift, bits=bits, pad=(ph, pw), algo=algo)
+        else:
+            got = qnn.conv_hwc(xd, wd, kd, ld_, bias=bd, shift=shift, bits=bits, stride=1, pad=(ph, pw), algo=algo)
+        qnn.device_status()
+        got = got.cpu().numpy().reshape(-1)
+        assert first_mismatch(got, want) is None, (seed, desc_str(n, h, w, c, m, kh, kw, ph, pw, bits, pool), algo,
+                                                   first_mismatch(got, want))
+
+
+def desc_str(*v):
+    return "n=%d h=%d w=%d c=%d m=%d k=%dx%d pad=%d,%d q%d pool=%d" % v
