@@ -273,6 +273,23 @@ int main()
     };
     for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 0);
     for (const auto &v : shapes) check(v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], 1);
+    // seeded random shapes across the planner's range (whatever it accepts is checked)
+    unsigned long long rng = 0x5EEDC0DEull;
+    auto next = [&](int lo, int hi) {  // uniform in [lo, hi]
+        rng = rng * 6364136223846793005ull + 1442695040888963407ull;
+        return lo + static_cast<int>((rng >> 33) % static_cast<unsigned long long>(hi - lo + 1));
+    };
+    static const int kBits[4] = {8, 8, 4, 2};
+    for (int i = 0; i < 300; ++i) {
+        const int bits = kBits[next(0, 3)];
+        const int per = 8 / bits;
+        const int c = per * next(1, bits == 8 ? 96 : 64);
+        const int m = per * next(1, 320 / per);
+        const int kh = next(1, 7), kw = next(1, 7);
+        const int ph = next(0, kh / 2), pw = next(0, kw / 2);
+        const int h = next(std::max(1, kh - 2 * ph), 40), w = next(std::max(1, kw - 2 * pw), 48);
+        check(next(1, 3), h, w, c, m, kh, kw, ph, pw, bits, next(0, 1));
+    }
     std::printf("fails=%d\n", fails);
     return fails != 0;
 }
