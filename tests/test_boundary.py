@@ -115,6 +115,35 @@ def test_conv_pointer_and_alignment_validation(lib):
     assert lib.qconv_hwc(None, *([None] * 8), ctypes.c_size_t(0), None) == qnn.QNN_EINVAL
 
 
+def test_prepare_and_run_validation(lib):
+    """qconv_hwc_prepare / qconv_hwc_run on the window kernel: the workspace (the prepared image,
+    qconv_hwc_workspace_size bytes, 256-byte aligned) is required by both; run needs x and y,
+    16-byte aligned; a descriptor that only the CUDA-core kernel takes has nothing to run.  No
+    CUDA call is reached."""
+    P, SZ = ctypes.c_void_p, ctypes.c_size_t
+    d = desc()
+    need = qnn.workspace_size(d)
+    assert need > 0
+
+    def prep(ws=FAKE, nbytes=need, w=FAKE, kappa=FAKE, lam=FAKE):
+        return lib.qconv_hwc_prepare(ctypes.byref(d), P(w), None, P(kappa), P(lam), None, P(ws), SZ(nbytes), None)
+
+    def run(dd=d, x=FAKE, y=FAKE, ws=FAKE, nbytes=need):
+        return lib.qconv_hwc_run(ctypes.byref(dd), P(x), P(y), P(ws), SZ(nbytes), None)
+
+    assert prep(ws=0) == qnn.QNN_EWORKSPACE
+    assert prep(nbytes=need - 1) == qnn.QNN_EWORKSPACE
+    assert prep(ws=FAKE + 16) == qnn.QNN_EWORKSPACE
+    assert prep(w=0) == qnn.QNN_EINVAL
+    assert prep(kappa=0) == qnn.QNN_EINVAL
+    assert run(ws=0) == qnn.QNN_EWORKSPACE
+    assert run(nbytes=need - 1) == qnn.QNN_EWORKSPACE
+    assert run(ws=FAKE + 128) == qnn.QNN_EWORKSPACE
+    assert run(x=0) == qnn.QNN_EINVAL
+    assert run(y=FAKE + 4) == qnn.QNN_EALIGN
+    assert run(dd=desc(stride=(2, 2))) == qnn.QNN_EUNSUPPORTED  # the CUDA-core kernel only
+
+
 def test_algo_selection_and_workspace(lib):
     assert qnn.conv_algo(desc()) == qnn.ALGO_TENSORCORE
     assert qnn.conv_algo(desc(stride=(2, 2))) == qnn.ALGO_DIRECT
